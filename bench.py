@@ -1,0 +1,407 @@
+"""Benchmark of the per-chunk revisit-consistency path on GB300.
+
+One step = one chunk step of the whole path on one batch of synthetic input:
+crc_cache_update -> crc_retrieve (score, top-k, gather) -> crc_correspond ->
+crc_biased_attention over all layers, at the Wan-1.3B chunk shape (12 heads,
+head dim 128, 30x52 tokens x 3 frames = 4680 queries, 18720 keys, bank of 64
+chunks, k = 1) with the 30 layers of one chunk step batched in one attention
+call.  Inputs are resident in HBM and far larger than L2 (K/V cache 3.4 GB).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config C] [--layers L]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
+
+Prints one JSON line.  `value` is the biased-attention algorithmic TFLOP/s of
+the whole step (4 N_q N_k d H L per step / step time, summed over ranks);
+per-stage GB/s for retrieval and reprojection ride along in `stages`.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "biased-attn TFLOP/s per chunk step (% of bf16 tensor peak); retrieve/reproj GB/s"
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"], src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ---------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------- workload
+def setup(cfg_id: int, layers: int, device: str, seed: int):
+    import torch
+
+    import synth
+    from paper_2607_21848_gb300 import api
+
+    wl = synth.make_workload(cfg_id, layers=layers)
+    dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    g = torch.Generator(device=device).manual_seed(seed)
+    s = wl.qkv_scale
+
+    def rnd(*shape):
+        return (torch.randn(*shape, generator=g, device=device) * s).to(dt)
+
+    Nc, L, H, d = wl.Nc, wl.L, wl.H, wl.d
+    W = dict(wl=wl, dtype=dt)
+    W["shape"] = api.shape(L, H, d, wl.F, wl.h, wl.w, dt)
+    bank = api.Bank(wl.bank_size + 1, wl.F, wl.h, wl.w, L, H, d, dt, wl.num_slabs, device=device)
+    api.crc_bank_insert_poses(bank, W["shape"], 0, synth.frame_records(wl.bank_frames))
+    bank.depth[:wl.bank_size] = torch.from_numpy(wl.depth_bank()).to(device)
+    for i in range(wl.num_slabs):
+        bank.kv[i, 0] = rnd(L, Nc, H, d)
+        bank.kv[i, 1] = rnd(L, Nc, H, d)
+    W["bank"] = bank
+    cache = api.Cache(rnd(L, wl.n_keys, H, d), rnd(L, wl.n_keys, H, d), wl.segments)
+    W["cache"] = cache
+    W["q"] = rnd(L, Nc, H, d)
+    W["o"] = torch.empty_like(W["q"])
+    W["k_new"] = rnd(L, Nc, H, d)
+    W["v_new"] = rnd(L, Nc, H, d)
+    W["depth"] = torch.from_numpy(wl.depth_of(wl.n)).to(device)
+    W["frames"] = synth.frame_records(wl.cur_frames)
+    W["idx"] = torch.zeros(wl.k, dtype=torch.int32, device=device)
+    W["score"] = torch.zeros(wl.k, dtype=torch.float64, device=device)
+    W["count"] = torch.zeros(1, dtype=torch.int32, device=device)
+    S = wl.k * wl.F
+    W["uv"] = torch.zeros(Nc, S, 2, device=device)
+    W["cell"] = torch.zeros(Nc, S, dtype=torch.int32, device=device)
+    W["valid"] = torch.zeros(Nc, S, dtype=torch.uint8, device=device)
+    W["status"] = torch.zeros(1, dtype=torch.int32, device=device)
+    W["params"] = api.retrieval_params(wl.E, wl.w_v, wl.tau_c, wl.cos_tau_v, wl.delta, wl.k, -1, 0)
+    # the current chunk enters the newest window slot
+    W["win_off"] = [off for off, _, kind, slot in wl.segments if kind == 2][-1]
+    return W
+
+
+def algorithmic(W):
+    """Algorithmic work of one step (what the method must do; padding not counted)."""
+    wl = W["wl"]
+    es = 2 if wl.dtype == "bf16" else 4
+    act_keys = sum(length for _, length, _, _ in wl.segments)
+    flops = 4.0 * wl.Nq * act_keys * wl.d * wl.H * wl.L
+    row = wl.H * wl.d * es
+    gather = 2 * 2 * wl.k * wl.L * wl.Nc * row  # K and V, read + write
+    score = wl.bank_size * 6 * 8
+    S = wl.k * wl.F
+    # reprojection: query depth, per pair u^ (8 B) + cell (4 B) + flag (1 B) + source depth lookup (4 B)
+    reproj = wl.Nq * 4 + wl.Nq * S * (8 + 4 + 1 + 4)
+    update = 2 * wl.L * wl.Nc * row * 3 + wl.Nc * 4 * 2  # read new K/V, write slab + window; depth
+    return dict(flops=flops, gather_bytes=gather + score, reproj_bytes=reproj, update_bytes=update)
+
+
+def run_step(W, stream, ev=None):
+    from paper_2607_21848_gb300 import api
+
+    wl = W["wl"]
+    if ev:
+        ev[0].record(stream)
+    api.crc_cache_update(W["bank"], W["shape"], wl.n, W["frames"], W["depth"], W["k_new"], W["v_new"], W["cache"],
+                         W["win_off"], stream)
+    if ev:
+        ev[1].record(stream)
+    api.crc_retrieve(W["bank"], wl.bank_size, W["shape"], W["frames"], wl.n, W["params"], W["cache"], W["idx"],
+                     W["score"], W["count"], stream)
+    if ev:
+        ev[2].record(stream)
+    api.crc_correspond(W["shape"], W["frames"], W["depth"], W["bank"], W["idx"], W["count"], wl.k, wl.eps, W["uv"],
+                       W["cell"], W["valid"], stream)
+    if ev:
+        ev[3].record(stream)
+    api.crc_biased_attention(W["shape"], W["q"], W["cache"], W["o"], None, W["uv"], W["valid"], wl.k, W["idx"],
+                             wl.lam, wl.sigma, 0, W["status"], stream)
+    if ev:
+        ev[4].record(stream)
+
+
+LAUNCHES_PER_STEP = 4
+
+
+# ---------------------------------------------------------------------------- oracle arm
+def oracle_sample(cfg_id: int, layers: int, budget_s: float):
+    """Time the fp64 oracle on a bounded sample of one step: the full retrieval and
+    correspondence, then attention rows of one head of one layer until `budget_s`."""
+    import oracle
+    import synth
+
+    wl = synth.make_workload(cfg_id, layers=1)
+    t0 = time.perf_counter()
+    bc = np.zeros((wl.bank_size, 3))
+    bv = np.zeros((wl.bank_size, 3))
+    for j in range(wl.bank_size):
+        bc[j], bv[j] = oracle.chunk_pose(wl.bank_frames.R[j], wl.bank_frames.c[j])
+    cn, vn = oracle.chunk_pose(wl.cur_frames.R, wl.cur_frames.c)
+    idx, _, count = oracle.retrieve(bc, bv, cn, vn, wl.n, wl.E, wl.w_v, wl.tau_c, wl.cos_tau_v, wl.delta, wl.k)
+    slots = oracle.fill_slots(idx, count, -1, 0)
+    S = wl.k * wl.F
+    Ks, Rs, cs = (np.zeros((S, 3, 3)), np.zeros((S, 3, 3)), np.zeros((S, 3)))
+    ds = np.ones((S, wl.h, wl.w), dtype=np.float32)
+    ok = np.zeros(S, bool)
+    for r, j in enumerate(slots):
+        for f in range(wl.F):
+            s = r * wl.F + f
+            fr = wl.bank_frames[max(j, 0)]
+            Ks[s], Rs[s], cs[s] = fr.K[f], fr.R[f], fr.c[f]
+            if j >= 0:
+                ds[s] = wl.depth_of(j)[f]
+                ok[s] = True
+    cur = wl.cur_frames
+    uv, _, valid = oracle.correspond(wl.depth_of(wl.n), cur.K, cur.R, cur.c, ds, Ks, Rs, cs, wl.eps, source_ok=ok)
+    t_front = time.perf_counter() - t0
+    g = np.random.default_rng(0)
+    Q = g.standard_normal((1, wl.Nq, 1, wl.d)) * wl.qkv_scale
+    Kc = g.standard_normal((1, wl.n_keys, 1, wl.d)) * wl.qkv_scale
+    Vc = g.standard_normal((1, wl.n_keys, 1, wl.d)) * wl.qkv_scale
+    act_keys = sum(length for _, length, _, _ in wl.segments)
+    rows_done, t_attn, blk = 0, 0.0, 256
+    while rows_done < wl.Nq and t_attn < budget_s:
+        rows = np.arange(rows_done, min(rows_done + blk, wl.Nq))
+        t1 = time.perf_counter()
+        oracle.attention(Q, Kc, Vc, uv, valid, wl.segments, wl.h, wl.w, wl.F, wl.lam, wl.sigma, slot_chunks=slots,
+                         rows=rows)
+        t_attn += time.perf_counter() - t1
+        rows_done += rows.shape[0]
+    flops_per_row = 4.0 * act_keys * wl.d  # one head, one layer
+    # one full step = L layers x H heads x Nq rows, plus one retrieval and one correspondence
+    step_s = t_front + t_attn / rows_done * wl.Nq * wl.H * layers
+    return dict(tflops=flops_per_row * rows_done / t_attn / 1e12, rows=rows_done, t_attn=t_attn, t_front=t_front,
+                step_s=step_s, threads=os.cpu_count())
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import synth
+
+    wl = synth.make_workload(args.config, layers=args.layers)
+    per_step = max(2.0, 60.0 / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        oracle_sample(args.config, args.layers, min(per_step, 2.0))
+    vals = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        vals.append(oracle_sample(args.config, args.layers, per_step))
+    el = time.perf_counter() - t0
+    tfl = statistics.median(v["tflops"] for v in vals)
+    sample = (f"per step: full retrieval over {wl.bank_size} chunks, full correspondence, and attention rows of "
+              f"one head of one layer for ~{per_step:.0f} s (median {statistics.median(v['rows'] for v in vals):.0f} "
+              f"of {wl.Nq} rows, all {wl.n_keys} keys); TFLOP/s = sampled attention FLOP / sampled time")
+    line = {"impl": "reference", "metric": METRIC, "value": tfl, "unit": "TFLOP/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": _config(wl, args),
+            "cpu_baseline": {"value": tfl, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": tfl, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def _config(wl, args):
+    return {"workload": f"{wl.name} chunk step: {wl.L} layers x {wl.H} heads, d={wl.d}, {wl.F}x{wl.h}x{wl.w} "
+                        f"queries={wl.Nq}, keys={wl.n_keys} (sink|{wl.k} retrieved|window), bank={wl.bank_size}, "
+                        f"k={wl.k}, lambda={wl.lam}, sigma={wl.sigma}",
+            "global_batch": args.gpus, "seq_len": wl.n_keys, "parallelism": f"{args.gpus} independent streams",
+            "l2": "inputs larger than L2 (no flush)"}
+
+
+# ---------------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--layers", type=int, default=30)
+    ap.add_argument("--impl", default="crc", choices=["crc", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    device = f"cuda:{local}"
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device(device))
+
+    from paper_2607_21848_gb300 import build
+
+    build.build()
+    W = setup(args.config, args.layers, device, seed=1234 + rank)
+    wl = W["wl"]
+    alg = algorithmic(W)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        run_step(W, stream)
+    barrier()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        barrier()
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for i in range(args.steps):
+            run_step(W, stream, evs[i])
+        t_end.record(stream)
+        barrier()
+    elapsed = t_start.elapsed_time(t_end) / 1e3
+    assert W["status"].item() == 0, "attention kernel reported a pipeline timeout"
+    if world > 1:
+        t = torch.tensor([elapsed], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    stage = {nm: statistics.median(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(args.steps)) / 1e3
+             for j, nm in enumerate(["update", "retrieve", "correspond", "attention"])}
+    step_s = elapsed / args.steps
+    value = alg["flops"] * world / step_s / 1e12
+
+    # end to end through the public API with host buffers: pinned inputs in, output out
+    host_in = {k: W[k].cpu().pin_memory() for k in ("q", "k_new", "v_new", "depth")}
+    host_out = torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True)
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + W["frames"].nbytes
+    d2h = host_out.numel() * host_out.element_size()
+    e2e_steps = max(3, min(args.steps, 20))
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        for k, t in host_in.items():
+            W[k].copy_(t, non_blocking=True)
+        run_step(W, stream)
+        host_out.copy_(W["o"], non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_s = e0.elapsed_time(e1) / 1e3 / e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_s], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    peaks = _peaks()
+    attn_tflops = alg["flops"] / stage["attention"] / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": _config(wl, args),
+        "stages": {
+            "update_ms": stage["update"] * 1e3, "update_gbs": alg["update_bytes"] / stage["update"] / 1e9,
+            "retrieve_ms": stage["retrieve"] * 1e3, "retrieve_gbs": alg["gather_bytes"] / stage["retrieve"] / 1e9,
+            "correspond_ms": stage["correspond"] * 1e3,
+            "correspond_gbs": alg["reproj_bytes"] / stage["correspond"] / 1e9,
+            "attention_ms": stage["attention"] * 1e3, "attention_tflops": attn_tflops,
+            "attention_frac_of_bf16_peak": attn_tflops / peaks["bf16_sus"],
+            "retrieve_frac_of_hbm_peak": alg["gather_bytes"] / stage["retrieve"] / 1e9 / peaks["hbm"],
+        },
+        "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel", "achieved": attn_tflops,
+                     "peak": peaks["bf16_sus"], "unit": "TFLOP/s", "frac": attn_tflops / peaks["bf16_sus"],
+                     "peak_source": f"{peaks['src']} bf16 sustained (kernel timed inside a long step)",
+                     "traffic": None},
+        "e2e": {"value": alg["flops"] * world / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h)},
+        "gpu_launches": LAUNCHES_PER_STEP * args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cb = oracle_sample(args.config, args.layers, 10.0)
+        line["cpu_baseline"] = {
+            "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["threads"], "kind": "oracle",
+            "sample": f"fp64 oracle: full retrieval + correspondence ({cb['t_front']:.2f} s), then {cb['rows']} of "
+                      f"{wl.Nq} attention rows of one head of one layer against all {wl.n_keys} keys "
+                      f"({cb['t_attn']:.1f} s); TFLOP/s = sampled attention FLOP / sampled time; a full step "
+                      f"extrapolates to {cb['step_s']:.0f} s"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

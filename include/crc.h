@@ -1,0 +1,265 @@
+/*
+ * crc.h — C ABI of the per-chunk revisit-consistency attention path.
+ *
+ * The path implements the inference-time method of "Closing the Loop:
+ * Training-Free Revisit Consistency for Autoregressive Generative Rendering":
+ *
+ *   crc_cache_update      Sec. 4.2  "Cache layout": the new chunk enters the recent
+ *                                   window; its K/V, depth and poses are retained
+ *                                   outside the attention cache (the memory bank).
+ *   crc_retrieve          Sec. 4.2, Eq. 1: score every historical chunk against the
+ *                                   current chunk's pose, gate, take the top-k, and
+ *                                   gather their K/V into the retrieved cache slots;
+ *                                   an empty admissible set extends the recent window.
+ *   crc_correspond        Sec. 4.3, Eq. 3-4: reproject each query token through its
+ *                                   depth and the relative pose into every retrieved
+ *                                   frame; visibility test; exact-fallback flags.
+ *   crc_biased_attention  Sec. 4.3, Eq. 2: softmax(q.k/sqrt(d) + lambda B) V, with the
+ *                                   Gaussian correspondence bias B computed inside the
+ *                                   tile loop on retrieved key columns only.
+ *
+ * Conventions shared by every entry point:
+ *   - All device pointers are caller-owned.  No entry point allocates or frees
+ *     memory; none keeps state between calls.
+ *   - Work is enqueued on the caller's stream `s`; results are valid once the
+ *     caller synchronises that stream.  No entry point synchronises the host,
+ *     except that host arrays passed by pointer are read before the call returns.
+ *   - Every argument is validated on the host before anything is enqueued; a
+ *     failed check returns an error code and enqueues nothing.
+ *   - Tensors of attention data use the token-major layout [L][N][H][d]
+ *     (layer, token, head, head-dim) with d contiguous; strides are in elements.
+ *   - Grid coordinates: token (row i, col j) of an h x w frame is the point
+ *     (x, y) = (j, i); tokens of a chunk are ordered frame, row, col.
+ */
+#ifndef CRC_H_
+#define CRC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes -------------------------------------------------------- */
+typedef int32_t crc_status;
+#define CRC_OK 0
+#define CRC_ERR_INVALID_ARG 1  /* null pointer, negative size, bad parameter value */
+#define CRC_ERR_SHAPE 2        /* inconsistent sizes or strides                   */
+#define CRC_ERR_UNSUPPORTED 3  /* dtype / head dim / alignment / device not handled */
+#define CRC_ERR_CUDA 4         /* a CUDA call failed; see crc_last_cuda_error()     */
+#define CRC_ERR_DEVICE 5       /* a kernel reported a failure in its status word    */
+
+/* ---- element types ------------------------------------------------------- */
+#define CRC_F32 0
+#define CRC_BF16 1
+
+/* ---- cache segment kinds (Sec. 4.2 "Cache layout") ----------------------- */
+#define CRC_SEG_SINK 0       /* the anchor: the first chunk, never evicted          */
+#define CRC_SEG_RETRIEVED 1  /* a pose-retrieved slot; `slot` = retrieval rank r    */
+#define CRC_SEG_WINDOW 2     /* the recent window (including the current chunk)     */
+
+#define CRC_MAX_SEGMENTS 16
+#define CRC_MAX_FRAMES 4   /* frames per chunk, F */
+#define CRC_MAX_K 8        /* retrieved slots per step, k */
+
+/* One latent frame's camera annotation (Sec. 4.1): intrinsics K rescaled to the
+ * token grid, camera-to-world rotation R and camera centre c, all row-major fp64.
+ * K must have last row (0, 0, 1). */
+typedef struct {
+  double K[9];
+  double R[9];
+  double c[3];
+} crc_frame;
+
+/* Problem shape of one call. */
+typedef struct {
+  int32_t L;      /* layers handled by the call                         */
+  int32_t H;      /* attention heads                                    */
+  int32_t d;      /* head dimension (64 or 128)                         */
+  int32_t F;      /* latent frames per chunk (1..CRC_MAX_FRAMES)         */
+  int32_t h, w;   /* token grid of one latent frame; N_c = F*h*w tokens */
+  int32_t dtype;  /* CRC_F32 or CRC_BF16                                 */
+} crc_shape;
+
+/* A [L][N][H][d] tensor: element (l, n, hd, e) is at
+ * data[l*stride_layer + n*stride_token + hd*stride_head + e]. */
+typedef struct {
+  void* data;
+  int64_t stride_layer;
+  int64_t stride_token;
+  int64_t stride_head;
+} crc_tensor;
+
+/* Contiguous key range [offset, offset+length) of the cache.  Keys outside every
+ * segment are masked.  A zero-length segment is allowed and contributes nothing. */
+typedef struct {
+  int32_t offset;
+  int32_t length;
+  int32_t kind;  /* CRC_SEG_* */
+  int32_t slot;  /* retrieval rank r for CRC_SEG_RETRIEVED (length must be N_c) */
+} crc_segment;
+
+/* The segmented clean KV cache [sink | retrieved slots | recent window]. */
+typedef struct {
+  crc_tensor k;  /* [L][n_keys][H][d]                                      */
+  crc_tensor v;  /* same layout and strides as k                           */
+  int32_t n_keys;
+  int32_t nseg;
+  crc_segment seg[CRC_MAX_SEGMENTS];
+} crc_cache;
+
+/* Memory bank of every chunk generated so far (Sec. 4.2: evicted chunks stay
+ * retrievable).  Device arrays, caller-allocated:
+ *   frames [capacity][F][21]  fp64 crc_frame records of every chunk
+ *   centre [capacity][3]      fp64 chunk centre c_j (written by the library)
+ *   view   [capacity][3]      fp64 unit view direction v_j (written by the library)
+ *   depth  [capacity][F][h][w] fp32 planar metric depth of every chunk
+ *   kv     [num_slabs][2][L][N_c][H][d] K (index 0) and V (index 1) slabs, dense,
+ *          dtype of the call; chunk j lives in slab j % num_slabs. */
+typedef struct {
+  int32_t capacity;
+  int32_t num_slabs;
+  double* frames;
+  double* centre;
+  double* view;
+  float* depth;
+  void* kv;
+} crc_bank;
+
+/* Eq. 1 parameters and the empty-set fallback of Sec. 4.2. */
+typedef struct {
+  double E;          /* scene-scale normaliser of the distance term (> 0)          */
+  double w_v;        /* weight of the angular term (0.5 in the paper)              */
+  double tau_c;      /* distance gate on ||c_j - c_n|| / E (may be +inf)           */
+  double cos_tau_v;  /* angle gate: admissible iff v_j . v_n >= cos_tau_v          */
+  int32_t delta;     /* temporal gap: admissible iff n - j >= delta                */
+  int32_t k;         /* retrieved slots (1..CRC_MAX_K)                             */
+  int32_t ext_first; /* fallback: slot r >= count holds chunk ext_first-(r-count)  */
+  int32_t ext_min;   /*   if that is >= ext_min (else the slot stays empty);       */
+                     /*   ext_first < 0 disables the fallback                      */
+} crc_retrieval;
+
+/* ---- library information ------------------------------------------------- */
+const char* crc_version(void);
+const char* crc_status_string(crc_status st);
+/* The cudaError_t of the last CRC_ERR_CUDA returned on this thread. */
+int32_t crc_last_cuda_error(void);
+
+/*
+ * crc_bank_insert_poses — record the camera annotations of chunks
+ * [first, first+count) in the bank and compute each chunk's centre and view
+ * direction (Sec. 4.2, the (c_j, v_j) of Eq. 1).
+ *
+ *   frames  host array [count][F] of crc_frame; copied to bank->frames.
+ * The chunk centre is the mean of its frames' centres and the view direction is
+ * the normalised sum of their optical axes (third column of R), in frame order,
+ * computed in fp64 without fused multiply-add.
+ * Errors: CRC_ERR_INVALID_ARG (null pointers, count < 0, first+count > capacity).
+ */
+crc_status crc_bank_insert_poses(const crc_bank* bank, const crc_shape* shape, int32_t first, int32_t count,
+                                 const crc_frame* frames, cudaStream_t s);
+
+/*
+ * crc_cache_update — Sec. 4.2 "Cache layout": chunk `chunk` (its K/V just
+ * produced by the clean-context pass) enters the recent window and the bank.
+ *
+ *   frames       host [F] crc_frame of the chunk; stored in the bank with its
+ *                centre and view direction (as crc_bank_insert_poses).
+ *   d_depth      device [F][h][w] fp32 depth; copied to bank->depth[chunk].
+ *   d_k, d_v     device [L][N_c][H][d] dense, dtype of the call; copied to slab
+ *                chunk % num_slabs of bank->kv and, if window_offset >= 0, to
+ *                cache keys [window_offset, window_offset + N_c) of every layer.
+ *                Both may be NULL (poses and depth only).
+ *   cache        may be NULL when window_offset < 0.
+ * The sink and the other cache keys are not touched.
+ * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE (window slot outside the cache),
+ * CRC_ERR_UNSUPPORTED (cache not dense per token), CRC_ERR_CUDA.
+ */
+crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_t chunk, const crc_frame* frames,
+                            const float* d_depth, const void* d_k, const void* d_v, const crc_cache* cache,
+                            int32_t window_offset, cudaStream_t s);
+
+/*
+ * crc_retrieve — Sec. 4.2, Eq. 1 over bank chunks j in [0, bank_count):
+ *   s(j) = ||c_j - c_n||_2 / E + w_v (1 - v_j . v_n)
+ *   A_n  = { j : ||c_j - c_n||/E <= tau_c, v_j . v_n >= cos_tau_v, n - j >= delta }
+ * where (c_n, v_n) summarise `cur` (host [F] frames of current chunk n) exactly as
+ * crc_bank_insert_poses does.  Scores are fp64 without FMA contraction, in the
+ * order dx*dx+dy*dy+dz*dz, sqrt, /E; dot product left to right.
+ *
+ * Outputs (device):
+ *   d_idx   [k] int32: the admissible chunks with the k smallest (s(j), j),
+ *           ascending; slots r >= count hold the window-extension chunk of
+ *           `p->ext_first` (or -1 when empty).
+ *   d_score [k] fp64: s(j) for r < count, +inf otherwise.  May be NULL.
+ *   d_count [1] int32: number of admissible chunks retrieved (<= k).
+ * Then, for every CRC_SEG_RETRIEVED segment of `cache` with slot r < k and
+ * d_idx[r] >= 0, keys [offset, offset+N_c) of every layer receive the K and V
+ * of slab d_idx[r] % num_slabs (the gather).  Everything stays on the device.
+ * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE, CRC_ERR_UNSUPPORTED, CRC_ERR_CUDA.
+ */
+crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
+                        int32_t n, const crc_retrieval* p, const crc_cache* cache, int32_t* d_idx, double* d_score,
+                        int32_t* d_count, cudaStream_t s);
+
+/*
+ * crc_correspond — Sec. 4.3, Eq. 3-4.  For every query token p = (t, i, j) of
+ * the current chunk and every source frame s = r*F + f of retrieved slot r < k:
+ *   X_t = z_p K_t^-1 (j, i, 1)^T,  X_s = R_s^T (R_t X_t + c_t - c_s),
+ *   u^  = pi(K_s X_s),  cell = (floor(u^x + 1/2), floor(u^y + 1/2)),
+ *   valid = z_p finite and > 0, u^ finite, [X_s]_z > 0, cell on the grid,
+ *           [X_s]_z <= (1 + eps) D_s(cell)  (eps = +inf disables Eq. 4),
+ *           d_idx[r] >= 0, and r < *d_count when d_count is not NULL
+ *           (a window-extension slot is not a retrieval and gets no bias).
+ * Source frames and depths are read from the bank at chunk d_idx[r] on the device.
+ * The per-pair transform is composed in fp64; per-token arithmetic is fp32.
+ *
+ *   cur      host [F] frames of the current chunk;  d_depth [F][h][w] fp32.
+ *   d_uv     device [N_q][S][2] fp32 u^ (NaN where undefined), S = k*F.
+ *   d_cell   device [N_q][S] int32: y*w + x, or -1 when not valid.  May be NULL.
+ *   d_valid  device [N_q][S] uint8: 1 valid, 0 not.
+ * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_CUDA.
+ */
+crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const float* d_depth, const crc_bank* bank,
+                          const int32_t* d_idx, const int32_t* d_count, int32_t k, float eps, float* d_uv,
+                          int32_t* d_cell, uint8_t* d_valid, cudaStream_t s);
+
+/* crc_biased_attention flags */
+#define CRC_ATTN_DEFAULT 0
+#define CRC_ATTN_SIMT 1  /* force the SIMT kernel (fp32 arithmetic) for any dtype */
+
+/*
+ * crc_biased_attention — Sec. 4.3, Eq. 2, for every layer l < L, head and query p:
+ *   A_pk = q_p . k_k / sqrt(d) + lambda B(p, k),  O_p = sum_k softmax_k(A_pk) v_k
+ *   B(p, k) = -||u_k - u^_s(p)||^2 / (2 sigma^2) when key k lies in a
+ *             CRC_SEG_RETRIEVED segment of slot r, s = r*F + (position in the
+ *             segment) / (h*w), u_k its (x, y) in that frame, and d_valid[p][s];
+ *             0 for every other key (sink, window) and for invalid pairs.
+ * Softmax runs over the active keys: keys inside a segment, minus retrieved slots
+ * whose chunk is empty (d_slot_chunk[r] < 0, when d_slot_chunk is not NULL).
+ * The bias is evaluated inside the tile loop and never stored.
+ *
+ *   q         [L][n_q][H][d] queries (dtype of the call); n_q = N_c.
+ *   o         [L][n_q][H][d] output, same dtype.
+ *   d_lse     device [L][H][n_q] fp32 natural-log sum-exp of the row, or NULL.
+ *   d_uv, d_valid   correspondences [n_q][S] from crc_correspond (S = k*F).
+ *   d_slot_chunk    device [k] int32 (crc_retrieve's d_idx) or NULL.
+ *   d_status  device int32 or NULL: set non-zero if a kernel gave up waiting on
+ *             an internal pipeline barrier (the output is then not valid).
+ * bf16 (d = 128) runs on the tcgen05 tensor-core kernel with fp32 softmax and
+ * accumulation; fp32 (or CRC_ATTN_SIMT) runs the SIMT kernel in fp32.
+ * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE, CRC_ERR_UNSUPPORTED (dtype, d,
+ * alignment, device without sm_103a), CRC_ERR_CUDA.
+ */
+crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_cache* cache, crc_tensor o,
+                                float* d_lse, int32_t n_q, const float* d_uv, const uint8_t* d_valid, int32_t k,
+                                const int32_t* d_slot_chunk, float lambda, float sigma, int32_t flags,
+                                int32_t* d_status, cudaStream_t s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CRC_H_ */

@@ -142,7 +142,7 @@ def reproject(u: np.ndarray, z: np.ndarray, Kt: np.ndarray, Rt: np.ndarray, ct: 
 
 def correspond(depth_t: np.ndarray, Kt: np.ndarray, Rt: np.ndarray, ct: np.ndarray,
                depth_s: np.ndarray, Ks: np.ndarray, Rs: np.ndarray, cs: np.ndarray,
-               eps: float, source_ok: Optional[np.ndarray] = None):
+               eps: float, source_ok: Optional[np.ndarray] = None, with_zs: bool = False):
     """Correspondence of every query token of the current chunk in every source frame.
 
     depth_t [F, h, w], Kt/Rt [F, 3, 3], ct [F, 3]: current (target) frames.
@@ -154,6 +154,7 @@ def correspond(depth_t: np.ndarray, Kt: np.ndarray, Rt: np.ndarray, ct: np.ndarr
     valid [Nq, S] bool, where valid means: the query depth is finite and positive,
     u-hat is finite, the point is in front of the source camera, the landing cell
     is on the grid, and Eq. 4 holds ([X_s]_z <= (1 + eps) D_s(cell)).
+    With `with_zs`, also returns [X_s]_z [Nq, S] (the point's depth in the source camera).
     """
     F, h, w = depth_t.shape
     S = depth_s.shape[0]
@@ -163,12 +164,14 @@ def correspond(depth_t: np.ndarray, Kt: np.ndarray, Rt: np.ndarray, ct: np.ndarr
     uv = np.zeros((Nq, S, 2))
     cell = np.full((Nq, S), -1, dtype=np.int32)
     valid = np.zeros((Nq, S), dtype=bool)
+    zs = np.zeros((Nq, S))
     for t in range(F):
         z = depth_t[t].astype(np.float64).ravel()
         rows = slice(t * h * w, (t + 1) * h * w)
         for s in range(S):
             u_hat, Xs = reproject(u, z, Kt[t], Rt[t], ct[t], Ks[s], Rs[s], cs[s])
             uv[rows, s] = u_hat
+            zs[rows, s] = Xs[:, 2]
             with np.errstate(invalid="ignore"):
                 cx = np.floor(u_hat[:, 0] + 0.5)
                 cy = np.floor(u_hat[:, 1] + 0.5)
@@ -183,6 +186,8 @@ def correspond(depth_t: np.ndarray, Kt: np.ndarray, Rt: np.ndarray, ct: np.ndarr
                 ok[:] = False
             valid[rows, s] = ok
             cell[rows, s] = np.where(ok, yi * w + xi, -1)
+    if with_zs:
+        return uv, cell, valid, zs
     return uv, cell, valid
 
 

@@ -1,0 +1,180 @@
+"""Python binding of the C ABI (argument marshalling only).
+
+Every function has the name of its C entry point and forwards to it; all
+arithmetic of the path runs in the CUDA kernels of libcrc.so.  PyTorch supplies
+device memory (tensors) and the current CUDA stream.  `Bank` and `Cache` are
+conveniences that allocate the caller-owned device buffers the C ABI expects.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import math
+from typing import Iterable, Optional, Sequence, Tuple
+
+import numpy as np
+import torch
+
+from . import _abi
+from ._abi import CrcError  # noqa: F401
+
+SEG_SINK = _abi.CRC_SEG_SINK
+SEG_RETRIEVED = _abi.CRC_SEG_RETRIEVED
+SEG_WINDOW = _abi.CRC_SEG_WINDOW
+ATTN_DEFAULT = _abi.CRC_ATTN_DEFAULT
+ATTN_SIMT = _abi.CRC_ATTN_SIMT
+
+
+def _dtype_code(dt: torch.dtype) -> int:
+    if dt == torch.float32:
+        return _abi.CRC_F32
+    if dt == torch.bfloat16:
+        return _abi.CRC_BF16
+    raise ValueError(f"unsupported dtype {dt}")
+
+
+def _stream(stream: Optional[torch.cuda.Stream]) -> C.c_void_p:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    return t.data_ptr()
+
+
+def shape(L: int, H: int, d: int, F: int, h: int, w: int, dtype: torch.dtype) -> _abi.crc_shape:
+    return _abi.crc_shape(L, H, d, F, h, w, _dtype_code(dtype))
+
+
+def frames_struct(records: np.ndarray):
+    """[N, 21] fp64 records (K 9, R 9, c 3) -> ctypes array of crc_frame."""
+    rec = np.ascontiguousarray(records, dtype=np.float64).reshape(-1, 21)
+    arr = (_abi.crc_frame * rec.shape[0])()
+    C.memmove(arr, rec.ctypes.data, rec.nbytes)
+    return arr
+
+
+def tensor_view(t: torch.Tensor) -> _abi.crc_tensor:
+    """crc_tensor of a [L, N, H, d] tensor with a contiguous last dimension."""
+    if t.dim() != 4 or t.stride(3) != 1:
+        raise ValueError("expected a [L, N, H, d] tensor with contiguous d")
+    return _abi.crc_tensor(_ptr(t), t.stride(0), t.stride(1), t.stride(2))
+
+
+class Bank:
+    """Device memory of the chunk bank (frames, pose summaries, depth, K/V slabs)."""
+
+    def __init__(self, capacity: int, F: int, h: int, w: int, L: int, H: int, d: int, dtype: torch.dtype,
+                 num_slabs: int, device="cuda", with_kv: bool = True):
+        self.capacity, self.F, self.h, self.w = capacity, F, h, w
+        self.L, self.H, self.d, self.dtype, self.num_slabs = L, H, d, dtype, num_slabs
+        self.frames = torch.zeros(capacity, F, 21, dtype=torch.float64, device=device)
+        self.centre = torch.zeros(capacity, 3, dtype=torch.float64, device=device)
+        self.view = torch.zeros(capacity, 3, dtype=torch.float64, device=device)
+        self.depth = torch.zeros(capacity, F, h, w, dtype=torch.float32, device=device)
+        self.kv = (torch.zeros(num_slabs, 2, L, F * h * w, H, d, dtype=dtype, device=device)
+                   if with_kv else None)
+
+    def struct(self) -> _abi.crc_bank:
+        return _abi.crc_bank(self.capacity, self.num_slabs, _ptr(self.frames), _ptr(self.centre), _ptr(self.view),
+                             _ptr(self.depth), _ptr(self.kv) if self.kv is not None else None)
+
+
+class Cache:
+    """Segmented clean KV cache [L, n_keys, H, d] with its segment table."""
+
+    def __init__(self, k: torch.Tensor, v: torch.Tensor, segments: Sequence[Tuple[int, int, int, int]]):
+        self.k, self.v = k, v
+        self.segments = [tuple(int(x) for x in s) for s in segments]
+
+    @classmethod
+    def empty(cls, L: int, n_keys: int, H: int, d: int, dtype: torch.dtype, segments, device="cuda"):
+        k = torch.zeros(L, n_keys, H, d, dtype=dtype, device=device)
+        v = torch.zeros_like(k)
+        return cls(k, v, segments)
+
+    @property
+    def n_keys(self) -> int:
+        return self.k.shape[1]
+
+    def struct(self) -> _abi.crc_cache:
+        c = _abi.crc_cache()
+        c.k = tensor_view(self.k)
+        c.v = tensor_view(self.v)
+        c.n_keys = self.n_keys
+        if len(self.segments) > _abi.CRC_MAX_SEGMENTS:
+            raise ValueError("too many segments")
+        c.nseg = len(self.segments)
+        for i, (off, length, kind, slot) in enumerate(self.segments):
+            c.seg[i] = _abi.crc_segment(off, length, kind, slot)
+        return c
+
+
+def retrieval_params(E: float, w_v: float, tau_c: float, cos_tau_v: float, delta: int, k: int,
+                     ext_first: int = -1, ext_min: int = 0) -> _abi.crc_retrieval:
+    return _abi.crc_retrieval(E, w_v, tau_c, cos_tau_v, delta, k, ext_first, ext_min)
+
+
+def crc_version() -> str:
+    return _abi.load().crc_version().decode()
+
+
+def crc_bank_insert_poses(bank: Bank, shp: _abi.crc_shape, first: int, frames: np.ndarray, stream=None) -> None:
+    lib = _abi.load()
+    fr = frames_struct(frames)
+    count = len(fr) // shp.F
+    b = bank.struct()
+    _abi.check("crc_bank_insert_poses",
+               lib.crc_bank_insert_poses(C.byref(b), C.byref(shp), first, count, fr, _stream(stream)))
+
+
+def crc_cache_update(bank: Bank, shp: _abi.crc_shape, chunk: int, frames: np.ndarray, depth: torch.Tensor,
+                     k_new: Optional[torch.Tensor], v_new: Optional[torch.Tensor], cache: Optional[Cache],
+                     window_offset: int, stream=None) -> None:
+    lib = _abi.load()
+    fr = frames_struct(frames)
+    b = bank.struct()
+    cs = cache.struct() if cache is not None else None
+    _abi.check("crc_cache_update",
+               lib.crc_cache_update(C.byref(b), C.byref(shp), chunk, fr, _ptr(depth), _ptr(k_new), _ptr(v_new),
+                                    C.byref(cs) if cs is not None else None, window_offset, _stream(stream)))
+
+
+def crc_retrieve(bank: Bank, bank_count: int, shp: _abi.crc_shape, cur_frames: np.ndarray, n: int,
+                 params: _abi.crc_retrieval, cache: Optional[Cache], idx: torch.Tensor, score: Optional[torch.Tensor],
+                 count: torch.Tensor, stream=None) -> None:
+    lib = _abi.load()
+    fr = frames_struct(cur_frames)
+    b = bank.struct()
+    cs = cache.struct() if cache is not None else None
+    _abi.check("crc_retrieve",
+               lib.crc_retrieve(C.byref(b), bank_count, C.byref(shp), fr, n, C.byref(params),
+                                C.byref(cs) if cs is not None else None, _ptr(idx), _ptr(score), _ptr(count),
+                                _stream(stream)))
+
+
+def crc_correspond(shp: _abi.crc_shape, cur_frames: np.ndarray, depth: torch.Tensor, bank: Bank, idx: torch.Tensor,
+                   count: Optional[torch.Tensor], k: int, eps: float, uv: torch.Tensor, cell: Optional[torch.Tensor],
+                   valid: torch.Tensor, stream=None) -> None:
+    lib = _abi.load()
+    fr = frames_struct(cur_frames)
+    b = bank.struct()
+    _abi.check("crc_correspond",
+               lib.crc_correspond(C.byref(shp), fr, _ptr(depth), C.byref(b), _ptr(idx), _ptr(count), k,
+                                  float(eps), _ptr(uv), _ptr(cell), _ptr(valid), _stream(stream)))
+
+
+def crc_biased_attention(shp: _abi.crc_shape, q: torch.Tensor, cache: Cache, o: torch.Tensor,
+                         lse: Optional[torch.Tensor], uv: Optional[torch.Tensor], valid: Optional[torch.Tensor], k: int,
+                         slot_chunk: Optional[torch.Tensor], lam: float, sigma: float, flags: int = 0,
+                         status: Optional[torch.Tensor] = None, stream=None) -> None:
+    lib = _abi.load()
+    cs = cache.struct()
+    _abi.check("crc_biased_attention",
+               lib.crc_biased_attention(C.byref(shp), tensor_view(q), C.byref(cs), tensor_view(o), _ptr(lse),
+                                        q.shape[1], _ptr(uv), _ptr(valid), k, _ptr(slot_chunk), float(lam),
+                                        float(sigma), flags, _ptr(status), _stream(stream)))

@@ -1,0 +1,334 @@
+// C ABI entry points: host-side argument validation, then one kernel launch each.
+#include <math.h>
+#include <string.h>
+
+#include "internal.cuh"
+
+namespace {
+
+thread_local int32_t g_last_cuda_error = 0;
+
+crc_status cuda_fail(cudaError_t e) {
+  g_last_cuda_error = (int32_t)e;
+  return CRC_ERR_CUDA;
+}
+
+int elem_bytes(int32_t dtype) { return dtype == CRC_BF16 ? 2 : 4; }
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+crc_status check_shape(const crc_shape* sh) {
+  if (!sh) return CRC_ERR_INVALID_ARG;
+  if (sh->L < 1 || sh->H < 1 || sh->F < 1 || sh->F > CRC_MAX_FRAMES || sh->h < 1 || sh->w < 1)
+    return CRC_ERR_INVALID_ARG;
+  if (sh->dtype != CRC_F32 && sh->dtype != CRC_BF16) return CRC_ERR_UNSUPPORTED;
+  if (sh->d < 8 || (sh->d % 8) != 0) return CRC_ERR_UNSUPPORTED;
+  const int64_t nc = (int64_t)sh->F * sh->h * sh->w;
+  if (nc > (1 << 24)) return CRC_ERR_SHAPE;
+  return CRC_OK;
+}
+
+bool frames_ok(const crc_frame* fr, int F) {
+  for (int f = 0; f < F; ++f) {
+    const double* K = fr[f].K;
+    if (K[6] != 0.0 || K[7] != 0.0 || K[8] != 1.0) return false;
+    for (int e = 0; e < 9; ++e)
+      if (!isfinite(fr[f].K[e]) || !isfinite(fr[f].R[e])) return false;
+    for (int e = 0; e < 3; ++e)
+      if (!isfinite(fr[f].c[e])) return false;
+  }
+  return true;
+}
+
+crc_status check_bank(const crc_bank* b, bool need_kv) {
+  if (!b || b->capacity < 1 || !b->frames || !b->centre || !b->view || !b->depth) return CRC_ERR_INVALID_ARG;
+  if (need_kv && (!b->kv || b->num_slabs < 1)) return CRC_ERR_INVALID_ARG;
+  return CRC_OK;
+}
+
+// The cache must hold whole token rows of H*d contiguous elements (stride_head = d,
+// stride_token >= H*d) with 16-byte aligned rows; k and v share strides.
+crc_status check_cache(const crc_cache* c, const crc_shape* sh) {
+  if (!c || !c->k.data || !c->v.data) return CRC_ERR_INVALID_ARG;
+  if (c->n_keys < 1 || c->nseg < 0 || c->nseg > CRC_MAX_SEGMENTS) return CRC_ERR_SHAPE;
+  if (c->k.stride_head != sh->d || c->k.stride_token < (int64_t)sh->H * sh->d ||
+      c->k.stride_layer < (int64_t)c->n_keys * c->k.stride_token)
+    return CRC_ERR_SHAPE;
+  if (c->v.stride_head != c->k.stride_head || c->v.stride_token != c->k.stride_token ||
+      c->v.stride_layer != c->k.stride_layer)
+    return CRC_ERR_SHAPE;
+  const int es = elem_bytes(sh->dtype);
+  if (!aligned16(c->k.data) || !aligned16(c->v.data) || (c->k.stride_token * es) % 16 != 0 ||
+      (c->k.stride_layer * es) % 16 != 0 || ((int64_t)sh->H * sh->d * es) % 16 != 0)
+    return CRC_ERR_UNSUPPORTED;
+  const int32_t nc = sh->F * sh->h * sh->w;
+  for (int g = 0; g < c->nseg; ++g) {
+    const crc_segment& s = c->seg[g];
+    if (s.offset < 0 || s.length < 0 || (int64_t)s.offset + s.length > c->n_keys) return CRC_ERR_SHAPE;
+    if (s.kind != CRC_SEG_SINK && s.kind != CRC_SEG_RETRIEVED && s.kind != CRC_SEG_WINDOW) return CRC_ERR_INVALID_ARG;
+    if (s.kind == CRC_SEG_RETRIEVED && (s.slot < 0 || s.slot >= CRC_MAX_K || (s.length != 0 && s.length != nc)))
+      return CRC_ERR_SHAPE;
+    for (int h2 = 0; h2 < g; ++h2) {  // segments may not overlap
+      const crc_segment& o = c->seg[h2];
+      if (s.length > 0 && o.length > 0 && s.offset < o.offset + o.length && o.offset < s.offset + s.length)
+        return CRC_ERR_SHAPE;
+    }
+  }
+  return CRC_OK;
+}
+
+void pack_frames(crc::FrameSet& fs, const crc_frame* fr, int F) {
+  memset(&fs, 0, sizeof(fs));
+  fs.F = F;
+  for (int f = 0; f < F; ++f) {
+    memcpy(&fs.rec[f][0], fr[f].K, 9 * sizeof(double));
+    memcpy(&fs.rec[f][9], fr[f].R, 9 * sizeof(double));
+    memcpy(&fs.rec[f][18], fr[f].c, 3 * sizeof(double));
+  }
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* crc_version(void) { return "crc 0.1.0 (sm_103a)"; }
+
+const char* crc_status_string(crc_status st) {
+  switch (st) {
+    case CRC_OK: return "ok";
+    case CRC_ERR_INVALID_ARG: return "invalid argument";
+    case CRC_ERR_SHAPE: return "inconsistent shape or stride";
+    case CRC_ERR_UNSUPPORTED: return "unsupported dtype, head dim, alignment or device";
+    case CRC_ERR_CUDA: return "CUDA error";
+    case CRC_ERR_DEVICE: return "kernel reported a failure";
+    default: return "unknown status";
+  }
+}
+
+int32_t crc_last_cuda_error(void) { return g_last_cuda_error; }
+
+crc_status crc_bank_insert_poses(const crc_bank* bank, const crc_shape* shape, int32_t first, int32_t count,
+                                 const crc_frame* frames, cudaStream_t s) {
+  crc_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_bank(bank, false))) return st;
+  if (count < 0 || first < 0 || (count > 0 && !frames)) return CRC_ERR_INVALID_ARG;
+  if ((int64_t)first + count > bank->capacity) return CRC_ERR_INVALID_ARG;
+  if (count == 0) return CRC_OK;
+  for (int32_t j = 0; j < count; ++j)
+    if (!frames_ok(frames + (int64_t)j * shape->F, shape->F)) return CRC_ERR_INVALID_ARG;
+  // crc_frame is exactly 21 packed doubles, the record layout of the bank
+  static_assert(sizeof(crc_frame) == crc::kFrameDoubles * sizeof(double), "crc_frame layout");
+  cudaError_t e = cudaMemcpyAsync(bank->frames + (int64_t)first * shape->F * crc::kFrameDoubles, frames,
+                                  (size_t)count * shape->F * sizeof(crc_frame), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  crc::PoseInsertArgs a{bank->frames, bank->centre, bank->view, shape->F, first, count};
+  e = crc::launch_pose_summary(a, s);
+  return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_t chunk, const crc_frame* frames,
+                            const float* d_depth, const void* d_k, const void* d_v, const crc_cache* cache,
+                            int32_t window_offset, cudaStream_t s) {
+  crc_status st = check_shape(shape);
+  if (st) return st;
+  const bool with_kv = d_k != nullptr || d_v != nullptr;
+  if ((st = check_bank(bank, with_kv))) return st;
+  if (!frames || !d_depth || chunk < 0 || chunk >= bank->capacity) return CRC_ERR_INVALID_ARG;
+  if ((d_k == nullptr) != (d_v == nullptr)) return CRC_ERR_INVALID_ARG;
+  if (!frames_ok(frames, shape->F)) return CRC_ERR_INVALID_ARG;
+  const int es = elem_bytes(shape->dtype);
+  const int32_t nc = shape->F * shape->h * shape->w;
+  const int32_t row_bytes = shape->H * shape->d * es;
+  if (with_kv && (!aligned16(d_k) || !aligned16(d_v) || !aligned16(bank->kv) || row_bytes % 16 != 0))
+    return CRC_ERR_UNSUPPORTED;
+  crc::CacheUpdateArgs a;
+  memset(&a, 0, sizeof(a));
+  pack_frames(a.frames, frames, shape->F);
+  a.bank_frames = bank->frames;
+  a.bank_centre = bank->centre;
+  a.bank_view = bank->view;
+  a.chunk = chunk;
+  a.depth_src = d_depth;
+  a.depth_count = nc;
+  a.depth_dst = bank->depth + (int64_t)chunk * nc;
+  a.L = shape->L;
+  a.Nc = nc;
+  a.row_bytes = row_bytes;
+  if (with_kv) {
+    a.k_src = static_cast<const char*>(d_k);
+    a.v_src = static_cast<const char*>(d_v);
+    const int64_t slab_bytes = 2LL * shape->L * nc * row_bytes;
+    a.slab = static_cast<char*>(bank->kv) + (int64_t)(chunk % bank->num_slabs) * slab_bytes;
+    if (window_offset >= 0) {
+      if ((st = check_cache(cache, shape))) return st;
+      if ((int64_t)window_offset + nc > cache->n_keys) return CRC_ERR_SHAPE;
+      a.win_k = static_cast<char*>(cache->k.data) + (int64_t)window_offset * cache->k.stride_token * es;
+      a.win_v = static_cast<char*>(cache->v.data) + (int64_t)window_offset * cache->v.stride_token * es;
+      a.win_layer_stride = cache->k.stride_layer * es;
+      a.win_token_stride = cache->k.stride_token * es;
+    }
+  }
+  cudaError_t e = crc::launch_cache_update(a, s);
+  return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
+                        int32_t n, const crc_retrieval* p, const crc_cache* cache, int32_t* d_idx, double* d_score,
+                        int32_t* d_count, cudaStream_t s) {
+  crc_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_bank(bank, cache != nullptr))) return st;
+  if (!cur || !p || !d_idx || !d_count) return CRC_ERR_INVALID_ARG;
+  if (bank_count < 0 || bank_count > bank->capacity) return CRC_ERR_INVALID_ARG;
+  if (p->k < 1 || p->k > CRC_MAX_K || !(p->E > 0.0) || isnan(p->w_v) || isnan(p->tau_c) || isnan(p->cos_tau_v))
+    return CRC_ERR_INVALID_ARG;
+  if (!frames_ok(cur, shape->F)) return CRC_ERR_INVALID_ARG;
+  crc::RetrieveArgs a;
+  memset(&a, 0, sizeof(a));
+  pack_frames(a.cur, cur, shape->F);
+  a.centre = bank->centre;
+  a.view = bank->view;
+  a.count = bank_count;
+  a.n = n;
+  a.E = p->E;
+  a.w_v = p->w_v;
+  a.tau_c = p->tau_c;
+  a.cos_tau_v = p->cos_tau_v;
+  a.delta = p->delta;
+  a.k = p->k;
+  a.ext_first = p->ext_first;
+  a.ext_min = p->ext_min;
+  a.d_idx = d_idx;
+  a.d_score = d_score;
+  a.d_count = d_count;
+  for (int r = 0; r < CRC_MAX_K; ++r) a.slot_offset[r] = -1;
+  if (cache) {
+    if ((st = check_cache(cache, shape))) return st;
+    const int es = elem_bytes(shape->dtype);
+    const int32_t nc = shape->F * shape->h * shape->w;
+    const int32_t row_bytes = shape->H * shape->d * es;
+    if (!aligned16(bank->kv)) return CRC_ERR_UNSUPPORTED;
+    a.pool = static_cast<const char*>(bank->kv);
+    a.num_slabs = bank->num_slabs;
+    a.layer_bytes = (int64_t)nc * row_bytes;
+    a.kv_bytes = (int64_t)shape->L * a.layer_bytes;
+    a.slab_bytes = 2 * a.kv_bytes;
+    a.cache_k = static_cast<char*>(cache->k.data);
+    a.cache_v = static_cast<char*>(cache->v.data);
+    a.cache_layer_stride = cache->k.stride_layer * es;
+    a.cache_token_stride = cache->k.stride_token * es;
+    a.L = shape->L;
+    a.Nc = nc;
+    a.row_bytes = row_bytes;
+    for (int g = 0; g < cache->nseg; ++g) {
+      const crc_segment& sg = cache->seg[g];
+      if (sg.kind == CRC_SEG_RETRIEVED && sg.slot < p->k && sg.length == nc) {
+        if (a.slot_offset[sg.slot] >= 0) return CRC_ERR_SHAPE;  // two segments for one slot
+        a.slot_offset[sg.slot] = sg.offset;
+      }
+    }
+  }
+  cudaError_t e = crc::launch_retrieve(a, s);
+  return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const float* d_depth, const crc_bank* bank,
+                          const int32_t* d_idx, const int32_t* d_count, int32_t k, float eps, float* d_uv,
+                          int32_t* d_cell, uint8_t* d_valid, cudaStream_t s) {
+  crc_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_bank(bank, false))) return st;
+  if (!cur || !d_depth || !d_idx || !d_uv || !d_valid) return CRC_ERR_INVALID_ARG;
+  if (k < 1 || k > CRC_MAX_K || isnan(eps) || eps < 0.f) return CRC_ERR_INVALID_ARG;
+  if (!frames_ok(cur, shape->F)) return CRC_ERR_INVALID_ARG;
+  if (((uintptr_t)d_uv & 7u) != 0) return CRC_ERR_UNSUPPORTED;
+  crc::CorrespondArgs a;
+  memset(&a, 0, sizeof(a));
+  pack_frames(a.cur, cur, shape->F);
+  a.depth = d_depth;
+  a.bank_frames = bank->frames;
+  a.bank_depth = bank->depth;
+  a.capacity = bank->capacity;
+  a.d_idx = d_idx;
+  a.d_count = d_count;
+  a.k = k;
+  a.F = shape->F;
+  a.h = shape->h;
+  a.w = shape->w;
+  a.eps = eps;
+  a.uv = d_uv;
+  a.cell = d_cell;
+  a.valid = d_valid;
+  cudaError_t e = crc::launch_correspond(a, s);
+  return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_cache* cache, crc_tensor o,
+                                float* d_lse, int32_t n_q, const float* d_uv, const uint8_t* d_valid, int32_t k,
+                                const int32_t* d_slot_chunk, float lambda, float sigma, int32_t flags,
+                                int32_t* d_status, cudaStream_t s) {
+  crc_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_cache(cache, shape))) return st;
+  if (!q.data || !o.data) return CRC_ERR_INVALID_ARG;
+  const int32_t nc = shape->F * shape->h * shape->w;
+  if (n_q != nc) return CRC_ERR_SHAPE;
+  if (k < 0 || k > CRC_MAX_K || !isfinite(lambda) || lambda < 0.f || !(sigma > 0.f) || !isfinite(sigma))
+    return CRC_ERR_INVALID_ARG;
+  bool any_ret = false;
+  for (int g = 0; g < cache->nseg; ++g)
+    if (cache->seg[g].kind == CRC_SEG_RETRIEVED && cache->seg[g].length > 0) {
+      any_ret = true;
+      if (cache->seg[g].slot >= k) return CRC_ERR_SHAPE;
+    }
+  if (any_ret && (!d_uv || !d_valid)) return CRC_ERR_INVALID_ARG;
+  if (q.stride_head < shape->d || q.stride_token < (int64_t)shape->H * q.stride_head ||
+      o.stride_head < shape->d || o.stride_token < (int64_t)shape->H * o.stride_head)
+    return CRC_ERR_SHAPE;
+  crc::AttnArgs a;
+  memset(&a, 0, sizeof(a));
+  a.q = q.data;
+  a.k = cache->k.data;
+  a.v = cache->v.data;
+  a.o = o.data;
+  a.lse = d_lse;
+  a.q_sl = q.stride_layer;
+  a.q_st = q.stride_token;
+  a.q_sh = q.stride_head;
+  a.k_sl = cache->k.stride_layer;
+  a.k_st = cache->k.stride_token;
+  a.k_sh = cache->k.stride_head;
+  a.o_sl = o.stride_layer;
+  a.o_st = o.stride_token;
+  a.o_sh = o.stride_head;
+  a.L = shape->L;
+  a.H = shape->H;
+  a.d = shape->d;
+  a.Nq = n_q;
+  a.Nk = cache->n_keys;
+  a.F = shape->F;
+  a.h = shape->h;
+  a.w = shape->w;
+  a.S = k * shape->F;
+  a.nseg = cache->nseg;
+  for (int g = 0; g < cache->nseg; ++g) a.seg[g] = cache->seg[g];
+  a.uv = d_uv;
+  a.valid = d_valid;
+  a.slot_chunk = d_slot_chunk;
+  a.lambda = lambda;
+  a.sigma = sigma;
+  a.dtype = shape->dtype;
+  a.status = d_status;
+  cudaError_t e;
+  if (shape->dtype == CRC_BF16 && !(flags & CRC_ATTN_SIMT)) {
+    e = crc::launch_attn_tc(a, s);
+    if (e == cudaErrorNotSupported) return CRC_ERR_UNSUPPORTED;
+  } else {
+    e = crc::launch_attn_simt(a, s);
+    if (e == cudaErrorNotSupported) return CRC_ERR_UNSUPPORTED;
+  }
+  return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+}  // extern "C"

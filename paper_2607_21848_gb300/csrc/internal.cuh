@@ -1,0 +1,147 @@
+// Internal declarations shared by the CUDA translation units of libcrc.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "crc.h"
+
+namespace crc {
+
+// One crc_frame record is 21 doubles: K[9], R[9], c[3].
+constexpr int kFrameDoubles = 21;
+
+struct FrameSet {
+  double rec[CRC_MAX_FRAMES][kFrameDoubles];
+  int32_t F;
+};
+
+// Chunk centre (mean of frame centres) and unit view direction (normalised sum of
+// optical axes, R[:, 2]) in fp64 with explicit round-to-nearest operations, so that
+// no multiply-add is ever contracted; summation runs in frame order.
+__device__ inline void chunk_summary(const double* rec, int F, double c[3], double v[3]) {
+  double c0 = rec[18], c1 = rec[19], c2 = rec[20];
+  double v0 = rec[9 + 2], v1 = rec[9 + 5], v2 = rec[9 + 8];
+  for (int f = 1; f < F; ++f) {
+    const double* r = rec + f * kFrameDoubles;
+    c0 = __dadd_rn(c0, r[18]);
+    c1 = __dadd_rn(c1, r[19]);
+    c2 = __dadd_rn(c2, r[20]);
+    v0 = __dadd_rn(v0, r[9 + 2]);
+    v1 = __dadd_rn(v1, r[9 + 5]);
+    v2 = __dadd_rn(v2, r[9 + 8]);
+  }
+  const double fF = (double)F;
+  c[0] = __ddiv_rn(c0, fF);
+  c[1] = __ddiv_rn(c1, fF);
+  c[2] = __ddiv_rn(c2, fF);
+  const double nrm = __dsqrt_rn(__dadd_rn(__dadd_rn(__dmul_rn(v0, v0), __dmul_rn(v1, v1)), __dmul_rn(v2, v2)));
+  v[0] = __ddiv_rn(v0, nrm);
+  v[1] = __ddiv_rn(v1, nrm);
+  v[2] = __ddiv_rn(v2, nrm);
+}
+
+// ---- launchers (defined in the kernel translation units) --------------------
+
+struct PoseInsertArgs {
+  double* frames;   // bank [capacity][F][21]
+  double* centre;   // bank [capacity][3]
+  double* view;     // bank [capacity][3]
+  int32_t F;
+  int32_t first;
+  int32_t count;
+};
+cudaError_t launch_pose_summary(const PoseInsertArgs& a, cudaStream_t s);
+
+struct CacheUpdateArgs {
+  FrameSet frames;
+  double* bank_frames;
+  double* bank_centre;
+  double* bank_view;
+  int32_t chunk;
+  const float* depth_src;  // [F][h][w]
+  float* depth_dst;        // bank depth + chunk * F*h*w
+  int32_t depth_count;
+  const char* k_src;       // [L][Nc][H][d] dense, or null
+  const char* v_src;
+  char* slab;              // bank kv slab of this chunk: [2][L][Nc][H][d]
+  char* win_k;             // cache k + window offset rows (layer 0), or null
+  char* win_v;
+  int64_t win_layer_stride;  // bytes
+  int64_t win_token_stride;  // bytes
+  int32_t L;
+  int32_t Nc;
+  int32_t row_bytes;       // H*d*elem
+};
+cudaError_t launch_cache_update(const CacheUpdateArgs& a, cudaStream_t s);
+
+struct RetrieveArgs {
+  FrameSet cur;
+  const double* centre;
+  const double* view;
+  int32_t count;
+  int32_t n;
+  double E, w_v, tau_c, cos_tau_v;
+  int32_t delta, k, ext_first, ext_min;
+  int32_t* d_idx;
+  double* d_score;
+  int32_t* d_count;
+  // gather (skipped when cache_k is null)
+  const char* pool;
+  int32_t num_slabs;
+  int64_t slab_bytes;
+  int64_t kv_bytes;     // bytes of the K half of a slab
+  int64_t layer_bytes;  // bytes of one layer inside a slab half
+  char* cache_k;
+  char* cache_v;
+  int64_t cache_layer_stride;  // bytes
+  int64_t cache_token_stride;  // bytes
+  int32_t slot_offset[CRC_MAX_K];  // token offset of slot r's segment, -1 if none
+  int32_t L;
+  int32_t Nc;
+  int32_t row_bytes;
+};
+cudaError_t launch_retrieve(const RetrieveArgs& a, cudaStream_t s);
+
+struct CorrespondArgs {
+  FrameSet cur;
+  const float* depth;        // [F][h][w]
+  const double* bank_frames; // [capacity][F][21]
+  const float* bank_depth;   // [capacity][F][h][w]
+  int32_t capacity;
+  const int32_t* d_idx;
+  const int32_t* d_count;    // may be null
+  int32_t k, F, h, w;
+  float eps;                 // +inf disables Eq. 4
+  float* uv;
+  int32_t* cell;             // may be null
+  uint8_t* valid;
+};
+cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s);
+
+struct AttnArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  void* o;
+  float* lse;
+  int64_t q_sl, q_st, q_sh;   // element strides
+  int64_t k_sl, k_st, k_sh;
+  int64_t o_sl, o_st, o_sh;
+  int32_t L, H, d, Nq, Nk;
+  int32_t F, h, w, S;
+  int32_t nseg;
+  crc_segment seg[CRC_MAX_SEGMENTS];
+  const float* uv;
+  const uint8_t* valid;
+  const int32_t* slot_chunk;
+  float lambda;
+  float sigma;
+  int32_t dtype;
+  int32_t* status;
+};
+cudaError_t launch_attn_simt(const AttnArgs& a, cudaStream_t s);
+// Returns cudaErrorNotSupported when the tensor-core kernel cannot take these arguments.
+cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s);
+
+}  // namespace crc

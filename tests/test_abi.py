@@ -1,0 +1,94 @@
+"""The C ABI library loads and exports every entry point include/crc.h declares,
+and the ctypes mirror has the C layout.  No compute call is made (no GPU here)."""
+
+import ctypes as C
+import os
+import re
+import shutil
+import subprocess
+import tempfile
+
+import pytest
+
+from paper_2607_21848_gb300 import _abi
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "crc.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\*?\s+\*?(crc_\w+)\s*\(", text, re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_21848_gb300 import build
+    build.build()
+    return _abi.load()
+
+
+def test_header_declares_the_four_path_calls():
+    names = _declared()
+    for n in ("crc_retrieve", "crc_correspond", "crc_biased_attention", "crc_cache_update"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert names
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(_abi.EXPORTED)
+    out = subprocess.run(["nm", "-D", "--defined-only", _abi.lib_path()], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (crc_\w+)", out))
+    assert set(names) <= exported
+
+
+def test_version_and_status_strings(lib):
+    assert "sm_103a" in lib.crc_version().decode()
+    for st in range(6):
+        assert lib.crc_status_string(st).decode()
+
+
+_LAYOUT_C = r"""
+#include <stdio.h>
+#include <stddef.h>
+#include "crc.h"
+#define P(T) printf(#T " %zu\n", sizeof(T));
+#define O(T, f) printf(#T "." #f " %zu\n", offsetof(T, f));
+int main(void) {
+  P(crc_frame) P(crc_shape) P(crc_tensor) P(crc_segment) P(crc_cache) P(crc_bank) P(crc_retrieval)
+  O(crc_cache, v) O(crc_cache, n_keys) O(crc_cache, seg) O(crc_bank, frames) O(crc_bank, kv)
+  O(crc_retrieval, delta) O(crc_retrieval, ext_min) O(crc_shape, dtype) O(crc_tensor, stride_head)
+  return 0;
+}
+"""
+
+
+def test_ctypes_layout_matches_header():
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    with tempfile.TemporaryDirectory() as td:
+        src = os.path.join(td, "layout.c")
+        exe = os.path.join(td, "layout")
+        open(src, "w").write(_LAYOUT_C)
+        r = subprocess.run([gcc, "-I", os.path.join(ROOT, "include"), "-I", "/usr/local/cuda/include", src, "-o", exe],
+                           capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
+        got = dict(line.rsplit(" ", 1) for line in subprocess.run([exe], capture_output=True, text=True).stdout.split("\n")
+                   if line)
+    ct = {
+        "crc_frame": C.sizeof(_abi.crc_frame), "crc_shape": C.sizeof(_abi.crc_shape),
+        "crc_tensor": C.sizeof(_abi.crc_tensor), "crc_segment": C.sizeof(_abi.crc_segment),
+        "crc_cache": C.sizeof(_abi.crc_cache), "crc_bank": C.sizeof(_abi.crc_bank),
+        "crc_retrieval": C.sizeof(_abi.crc_retrieval),
+        "crc_cache.v": _abi.crc_cache.v.offset, "crc_cache.n_keys": _abi.crc_cache.n_keys.offset,
+        "crc_cache.seg": _abi.crc_cache.seg.offset, "crc_bank.frames": _abi.crc_bank.frames.offset,
+        "crc_bank.kv": _abi.crc_bank.kv.offset, "crc_retrieval.delta": _abi.crc_retrieval.delta.offset,
+        "crc_retrieval.ext_min": _abi.crc_retrieval.ext_min.offset, "crc_shape.dtype": _abi.crc_shape.dtype.offset,
+        "crc_tensor.stride_head": _abi.crc_tensor.stride_head.offset,
+    }
+    for k, v in ct.items():
+        assert int(got[k]) == v, (k, got[k], v)

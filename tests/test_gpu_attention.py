@@ -1,0 +1,182 @@
+"""GPU parity of the biased attention (Eq. 2) against the fp64 oracle.
+
+fp32 path: max abs error <= 1e-4.  bf16 path (tcgen05 kernel): max abs error
+<= 2e-2 and, because the synthetic workloads have small outputs, also max abs
+error <= 2e-2 x RMS(O_oracle); LSE within 1e-3.  Both sides receive the same
+correspondences (the oracle's, rounded to fp32) so that attention is compared
+on identical inputs."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from paper_2607_21848_gb300 import api
+from tests import _gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2607_21848_gb300 import build
+    build.build()
+
+
+def _run_attn(shp, Q, Kc, Vc, segs, uv, valid, k, lam, sigma, slot_chunk=None, flags=0, dtype=torch.bfloat16):
+    q = Q if isinstance(Q, torch.Tensor) else _gpu.to_dev(Q, dtype)
+    cache = api.Cache(Kc if isinstance(Kc, torch.Tensor) else _gpu.to_dev(Kc, dtype),
+                      Vc if isinstance(Vc, torch.Tensor) else _gpu.to_dev(Vc, dtype), segs)
+    o = torch.full_like(q, float("nan"))
+    L, Nq, H, _ = q.shape
+    lse = torch.full((L, H, Nq), float("nan"), device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    uvt = _gpu.to_dev(uv.astype(np.float32)) if uv is not None else None
+    vt = _gpu.to_dev(valid.astype(np.uint8)) if valid is not None else None
+    sc = _gpu.to_dev(np.asarray(slot_chunk, dtype=np.int32)) if slot_chunk is not None else None
+    api.crc_biased_attention(shp, q, cache, o, lse, uvt, vt, k, sc, lam, sigma, flags, status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    return o.float().cpu().numpy(), lse.cpu().numpy()
+
+
+def _small_case(seed=0, L=2, H=2, F=3, h=12, w=16, k=2, window=2, scale=1.0, p_valid=0.7):
+    g = np.random.default_rng(seed)
+    Nc = F * h * w
+    segs = [(0, Nc, api.SEG_SINK, 0)] + [((1 + r) * Nc, Nc, api.SEG_RETRIEVED, r) for r in range(k)] + \
+           [((1 + k + q) * Nc, Nc, api.SEG_WINDOW, q) for q in range(window)]
+    Nk = (1 + k + window) * Nc
+    bf = lambda a: synth.bf16_round(a.astype(np.float32) * scale)  # noqa: E731
+    Q = bf(g.standard_normal((L, Nc, H, 128)))
+    Kc = bf(g.standard_normal((L, Nk, H, 128)))
+    Vc = bf(g.standard_normal((L, Nk, H, 128)))
+    S = k * F
+    uv = np.stack([g.uniform(-1.0, w, size=(Nc, S)), g.uniform(-1.0, h, size=(Nc, S))], -1).astype(np.float32)
+    valid = g.uniform(size=(Nc, S)) < p_valid
+    shp = api.shape(L, H, 128, F, h, w, torch.bfloat16)
+    return shp, Q, Kc, Vc, segs, uv, valid, (F, h, w, k)
+
+
+def _oracle(Q, Kc, Vc, uv, valid, segs, geom, lam, sigma, slot_chunk=None, **kw):
+    F, h, w, k = geom
+    return oracle.attention(Q, Kc, Vc, uv.astype(np.float64), valid, segs, h, w, F, lam, sigma,
+                            slot_chunks=None if slot_chunk is None else np.asarray(slot_chunk), **kw)
+
+
+def _check_bf16(Og, lg, Oo, lo, rows=None):
+    if rows is not None:
+        Og = Og[:, rows]
+    err, rel, rms = _gpu.attn_errors(Og, Oo)
+    assert err <= 2e-2, (err, rms)
+    assert rel <= 2e-2, (err, rel, rms)
+    if lg is not None:
+        lg = lg if rows is None else lg[:, :, rows]
+        assert np.abs(lg - lo).max() <= 1e-3
+
+
+def test_fp32_config1_matches_oracle_1e4():
+    wl = synth.make_workload(1)
+    idx, _, count, slots = _gpu.oracle_retrieve(wl)
+    uv, cell, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
+    assert valid.any()
+    Q, Kc, Vc = synth.make_qkv(wl)
+    shp = api.shape(wl.L, wl.H, wl.d, wl.F, wl.h, wl.w, torch.float32)
+    Og, lg = _run_attn(shp, Q, Kc, Vc, wl.segments, uv.astype(np.float32), valid, wl.k, wl.lam, wl.sigma,
+                       slot_chunk=slots, dtype=torch.float32)
+    Oo, lo = oracle.attention(Q, Kc, Vc, uv.astype(np.float32).astype(np.float64), valid, wl.segments, wl.h, wl.w,
+                              wl.F, wl.lam, wl.sigma, slot_chunks=slots)
+    assert np.abs(Og - Oo).max() <= 1e-4
+    assert np.abs(lg - lo).max() <= 1e-4
+    # the bias matters here: without it the output moves well beyond the tolerance
+    O0, _ = oracle.attention(Q, Kc, Vc, uv, valid, wl.segments, wl.h, wl.w, wl.F, 0.0, wl.sigma)
+    assert np.abs(O0 - Oo).max() > 1e-2
+
+
+@pytest.mark.parametrize("lam,sigma", [(0.0, 1.0), (2.0, 1.0), (8.0, 0.5)])
+def test_bf16_tcgen05_small_ragged(lam, sigma):
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case()
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], lam, sigma)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, lam, sigma)
+    _check_bf16(Og, lg, Oo, lo)
+
+
+def test_bf16_simt_path_matches_oracle():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=1, L=1)
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=api.ATTN_SIMT)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0)
+    _check_bf16(Og, lg, Oo, lo)
+
+
+def test_bf16_all_invalid_equals_lambda_zero_bitwise():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=2)
+    O0, l0 = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 0.0, 1.0)
+    O1, l1 = _run_attn(shp, Q, Kc, Vc, segs, uv, np.zeros_like(valid), geom[3], 5.0, 0.7)
+    np.testing.assert_array_equal(O0, O1)
+    np.testing.assert_array_equal(l0, l1)
+
+
+def test_bf16_empty_slot_and_short_segments_are_masked():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=3, k=2, window=2)
+    F, h, w, k = geom
+    Nc = F * h * w
+    # slot 1 empty; second window slot holds only 100 keys; sink shortened to 300 keys
+    segs2 = [(0, 300, api.SEG_SINK, 0), segs[1], segs[2], segs[3], (segs[4][0], 100, api.SEG_WINDOW, 1)]
+    slot_chunk = [4, -1]
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs2, uv, valid, k, 2.0, 1.0, slot_chunk=slot_chunk)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs2, geom, 2.0, 1.0, slot_chunk=slot_chunk)
+    _check_bf16(Og, lg, Oo, lo)
+
+
+def test_bf16_no_active_key_gives_zero_output():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=4, L=1, H=1)
+    F, h, w, k = geom
+    segs2 = [(segs[1][0], segs[1][1], api.SEG_RETRIEVED, 0)]
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs2, uv, valid, k, 2.0, 1.0, slot_chunk=[-1, -1])
+    assert np.all(Og == 0) and np.all(np.isneginf(lg))
+
+
+def _full_size(cfg, rows, layers, heads, seed=7):
+    wl = synth.make_workload(cfg)
+    _, _, count, slots = _gpu.oracle_retrieve(wl)
+    uv, _, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
+    uv = uv.astype(np.float32)
+    uv[~valid] = 0.0
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    s = wl.qkv_scale
+    q = (torch.randn(wl.L, wl.Nq, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    kc = (torch.randn(wl.L, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    vc = (torch.randn(wl.L, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    shp = api.shape(wl.L, wl.H, wl.d, wl.F, wl.h, wl.w, torch.bfloat16)
+    Og, lg = _run_attn(shp, q, kc, vc, wl.segments, uv, valid, wl.k, wl.lam, wl.sigma, slot_chunk=slots)
+    Lsel, Hsel = list(layers), list(heads)
+    Qo = q[Lsel][:, :, Hsel].float().cpu().numpy()
+    Ko = kc[Lsel][:, :, Hsel].float().cpu().numpy()
+    Vo = vc[Lsel][:, :, Hsel].float().cpu().numpy()
+    Oo, lo = oracle.attention(Qo, Ko, Vo, uv.astype(np.float64), valid, wl.segments, wl.h, wl.w, wl.F, wl.lam,
+                              wl.sigma, slot_chunks=slots, rows=rows)
+    Og = Og[Lsel][:, :, Hsel]
+    lg = lg[Lsel][:, Hsel]
+    _check_bf16(Og, lg, Oo, lo, rows=rows)
+    # the correspondence bias changes the output by far more than the tolerance
+    assert valid.mean() > 0.05
+
+
+def test_bf16_config2_full_size_sampled_rows():
+    rows = np.random.default_rng(0).choice(4680, 1024, replace=False)
+    rows.sort()
+    _full_size(2, rows, [0], range(12))
+
+
+def test_bf16_config3_30_layers_sampled():
+    rows = np.random.default_rng(1).choice(4680, 256, replace=False)
+    rows.sort()
+    _full_size(3, rows, [0, 17, 29], [0, 5, 11])
+
+
+def test_bf16_config4_full_size_sampled():
+    rows = np.random.default_rng(2).choice(10800, 256, replace=False)
+    rows.sort()
+    _full_size(4, rows, [0], [0, 13, 39])

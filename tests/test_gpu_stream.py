@@ -1,0 +1,110 @@
+"""The long-horizon loop-closure stream (200 chunk steps on a closed camera loop,
+Wan-1.3B head shape, 30 layers, k = 2) through ChunkStream: every step's
+retrieval must match the oracle bit-exactly and its correspondences within the
+boundary band; the cache invariants (sink = chunk 0, window = newest chunks,
+retrieved slots = their slabs) must hold; attention is compared with the oracle on
+sampled steps, layers and query rows."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from paper_2607_21848_gb300 import stream as crs
+from tests import _gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2607_21848_gb300 import build
+    build.build()
+
+
+def test_loop_stream_200_steps():
+    wl = synth.make_workload(5)
+    cfg = crs.StreamConfig(L=wl.L, H=wl.H, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2,
+                           capacity=wl.bank_size, num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c,
+                           cos_tau_v=wl.cos_tau_v, delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps)
+    st = crs.ChunkStream(cfg)
+    Nc = cfg.Nc
+    g = torch.Generator(device="cuda").manual_seed(5)
+    s = wl.qkv_scale
+    nbuf = 3
+    kv_new = [((torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device="cuda") * s).bfloat16(),
+               (torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device="cuda") * s).bfloat16()) for _ in range(nbuf)]
+    q = (torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device="cuda") * s).bfloat16()
+    o = torch.empty_like(q)
+    lse = torch.empty(cfg.L, cfg.H, Nc, device="cuda")
+    check_attn = {1, 2, 3, 150, 151, 199}
+    layers, heads = [0, 29], [0, 7]
+    host_kv = [(kb[layers][:, :, heads].double().cpu().numpy(), vb[layers][:, :, heads].double().cpu().numpy())
+               for kb, vb in kv_new]
+    host_q = q[layers][:, :, heads].double().cpu().numpy()
+
+    def slab_owner(slab, n):
+        """Newest chunk m <= n written to K/V slab `slab` (chunk m lives in slab m % P)."""
+        return slab + ((n - slab) // cfg.num_slabs) * cfg.num_slabs
+    n_closed = 0
+    for n in range(wl.bank_size):
+        fr = wl.bank_frames[n]
+        dep = torch.from_numpy(wl.depth_of(n)).cuda()
+        kn, vn = kv_new[n % nbuf]
+        st.step(n, synth.frame_records(fr), dep, kn, vn, q, o, lse)
+        torch.cuda.synchronize()
+        assert st.status.item() == 0
+        # retrieval: bit-exact indices and count
+        ext = st.ext_first(n)
+        oi, os_, oc, slots = _gpu.oracle_retrieve(wl, bank_count=n + 1, n=n, ext_first=ext, ext_min=1)
+        gi = st.idx.cpu().numpy()
+        assert int(st.count.item()) == oc, n
+        np.testing.assert_array_equal(gi, slots)
+        np.testing.assert_array_equal(st.score.cpu().numpy()[:oc], os_[:oc])
+        n_closed += oc > 0
+        # cache invariants, against the chunks' K/V buffers
+        assert torch.equal(st.cache.k[:, :Nc], kv_new[0][0])  # sink = chunk 0
+        for m in range(max(1, n - 1), n + 1):
+            off = st.window_offset(m % 2)
+            assert torch.equal(st.cache.k[:, off:off + Nc], kv_new[m % nbuf][0])
+            assert torch.equal(st.cache.v[:, off:off + Nc], kv_new[m % nbuf][1])
+        for r, j in enumerate(slots):
+            if j >= 0:
+                off = st.slot_offset(r)
+                src = kv_new[slab_owner(j % cfg.num_slabs, n) % nbuf]
+                assert torch.equal(st.cache.k[:, off:off + Nc], src[0])
+                assert torch.equal(st.cache.v[:, off:off + Nc], src[1])
+        # correspondences
+        ocor = _gpu.oracle_correspond(wl, slots, oc, cur=fr, depth_cur=wl.depth_of(n))
+        r = _gpu.compare_correspondence(wl, ocor, st.uv.cpu().numpy().astype(np.float64), st.cell.cpu().numpy(),
+                                        st.valid.cpu().numpy(), wl.eps, depth_cur=wl.depth_of(n))
+        assert r["bad_valid"] == 0 and r["bad_cell"] == 0 and r["uv_err"] <= 1e-3, (n, r)
+        if n in check_attn:
+            # oracle inputs come from the seeded inputs only: its own retrieval and
+            # correspondences, and a cache assembled from the chunks' K/V buffers
+            uv, _, valid, _, _, _ = ocor
+            agree = (st.valid.cpu().numpy().astype(bool) == valid).all(axis=1)
+            rows = np.random.default_rng(n).choice(np.nonzero(agree)[0], 128, replace=False)
+            rows.sort()
+            Kx = np.zeros((len(layers), cfg.n_keys, len(heads), cfg.d))
+            Vx = np.zeros_like(Kx)
+            Kx[:, :Nc], Vx[:, :Nc] = host_kv[0]
+            for rr, j in enumerate(slots):
+                if j >= 0:
+                    off = st.slot_offset(rr)
+                    Kx[:, off:off + Nc], Vx[:, off:off + Nc] = host_kv[slab_owner(j % cfg.num_slabs, n) % nbuf]
+            for m in range(max(1, n - 1), n + 1):
+                off = st.window_offset(m % 2)
+                Kx[:, off:off + Nc], Vx[:, off:off + Nc] = host_kv[m % nbuf]
+            uvo = uv.copy()
+            uvo[~valid] = 0.0
+            Oo, lo = oracle.attention(host_q, Kx, Vx, uvo.astype(np.float32).astype(np.float64), valid,
+                                      st.segments(n), cfg.h, cfg.w, cfg.F, cfg.lam, cfg.sigma, slot_chunks=slots,
+                                      rows=rows)
+            Og = o[layers][:, :, heads].float().cpu().numpy()[:, rows]
+            err, rel, rms = _gpu.attn_errors(Og, Oo)
+            assert err <= 2e-2 and rel <= 2e-2, (n, err, rel)
+            lg = lse[layers][:, heads].cpu().numpy()[:, :, rows]
+            assert np.abs(lg - lo).max() <= 1e-3
+    assert n_closed >= 40  # the loop closes after one lap and stays closed
