@@ -12,6 +12,7 @@
 //   warp  8    TMA producer: Q once, then K/V tiles of 128 keys, 2 stages each,
 //              128-byte swizzled boxes of 128 rows x 64 elements
 //   warp  9    TMEM owner and single-thread tcgen05.mma issuer
+//   warps 10-11 idle (they complete the third warpgroup for the register split)
 // TMEM (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each.  S = Q K^T is an
 // SS MMA (both operands K-major in shared memory); each softmax thread reads its
 // row of S, writes P in bf16 over the first 64 columns of the same S buffer and
@@ -42,9 +43,15 @@ constexpr int BN = 128;  // keys per KV tile
 constexpr int HD = 128;  // head dim
 constexpr int NQT = 2;   // query tiles per CTA
 constexpr int ST = 2;    // stages for K and for V
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;  // 3 warpgroups: softmax 0, softmax 1, producer/MMA
 constexpr int kWarpTma = 8;
 constexpr int kWarpMma = 9;
+// register split (setmaxnreg): the block launches with 384 x 168 registers; the
+// producer warpgroup drops to 96 and each softmax warpgroup rises to 200:
+// 2 x 128 x 200 + 128 x 96 <= 384 x 168.
+constexpr int kRegsSoftmax = 200;
+constexpr int kRegsProducer = 96;
+static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * 168, "register split exceeds the launch");
 constexpr int BOX = BM * 64 * 2;  // 128 rows x 64 bf16 = 16 KB
 constexpr int TILE = 2 * BOX;     // 128 rows x 128 bf16 = 32 KB
 constexpr int kMaxTiles = 1024;   // KV tiles per call
@@ -65,7 +72,8 @@ constexpr uint32_t TM_O = 256;  // O of tile x at column 256 + 128 x
 constexpr uint32_t TM_COLS = 512;
 
 constexpr uint8_t CLS_PLAIN = 0;    // every column active, none biased
-constexpr uint8_t CLS_GENERAL = 1;  // bias and/or masked columns
+constexpr uint8_t CLS_BIAS1 = 1;    // every column active and biased, one source frame
+constexpr uint8_t CLS_GENERAL = 2;  // anything else: per-column bias / mask
 
 struct TileInfo {
   uint16_t tile;
@@ -91,6 +99,70 @@ __device__ __forceinline__ int B_SFULL(int x) { return 1 + 4 * ST + x; }
 __device__ __forceinline__ int B_PREADY(int x) { return 1 + 4 * ST + NQT + x; }
 __device__ __forceinline__ int B_OFINAL(int x) { return 1 + 4 * ST + 2 * NQT + x; }
 __device__ __forceinline__ int B_DRAIN() { return 1 + 4 * ST + 3 * NQT; }
+
+// ---- packed fp32 pairs (Blackwell f32x2 ALU ops) and three-input max ----------
+__device__ __forceinline__ uint64_t pk2(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t fsub2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// One query row's correspondences in the two source frames of a KV tile, with the
+// bias coefficient already zero for invalid pairs (exact fallback).
+struct Corr {
+  float uxA, uyA, cA, uxB, uyB, cB;
+};
+
+__device__ __forceinline__ Corr load_corr(const AttnArgs& a, const TileInfo* tiles, int j, int nt, int p, bool row_ok,
+                                          float coef) {
+  Corr c{0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (j >= nt || !row_ok) return c;
+  const TileInfo ti = tiles[j];
+  if (ti.sA < 0) return c;
+  const int64_t ia = (int64_t)p * a.S + ti.sA, ib = (int64_t)p * a.S + ti.sB;
+  const float2* uv = reinterpret_cast<const float2*>(a.uv);
+  if (__ldg(a.valid + ia)) {
+    const float2 u = __ldg(uv + ia);
+    c.uxA = u.x;
+    c.uyA = u.y;
+    c.cA = coef;
+  }
+  if (__ldg(a.valid + ib)) {
+    const float2 u = __ldg(uv + ib);
+    c.uxB = u.x;
+    c.uyB = u.y;
+    c.cB = coef;
+  }
+  return c;
+}
 
 __device__ __forceinline__ void fail(const TcParams& P, volatile int* abort_flag, int code) {
   *abort_flag = 1;
@@ -147,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ti.sB = -1;
       if (t < ntot) {
         const int k0 = t * BN, k1 = k0 + BN;
-        int nact = 0, sA = 1 << 20, sB = -1;
+        int nact = 0, nbias = 0, sA = 1 << 20, sB = -1;
         for (int g = 0; g < a.nseg; ++g) {
           const crc_segment sg = a.seg[g];
           if (sg.length <= 0) continue;
@@ -157,6 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (a.slot_chunk && a.slot_chunk[sg.slot] < 0) continue;
             sA = min(sA, sg.slot * a.F + (lo - sg.offset) / hw);
             sB = max(sB, sg.slot * a.F + (hi - 1 - sg.offset) / hw);
+            nbias += hi - lo;
           }
           nact += hi - lo;
         }
@@ -165,7 +238,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           ti.sA = (int8_t)sA;
           ti.sB = (int8_t)sB;
         }
-        ti.cls = (nact == BN && sB < 0) ? CLS_PLAIN : CLS_GENERAL;
+        ti.cls = (nact == BN && sB < 0) ? CLS_PLAIN
+                 : (nact == BN && nbias == BN && sA == sB) ? CLS_BIAS1 : CLS_GENERAL;
       }
       const unsigned m = __ballot_sync(0xffffffffu, act);
       if (act) tiles[count + __popc(m & ((1u << lane) - 1u))] = ti;
@@ -184,7 +258,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nt = *ntiles_slot;
   const uint64_t T = P.timeout_ns;
 
-  if (warp == kWarpTma) {
+  if (warp >= 8) {
+   asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsProducer));
+   if (warp == kWarpTma) {
     // ------------------------------------------------------------ producer
     if (lane == 0 && nt > 0) {
       prefetch_tensormap(&tmQ);
@@ -221,26 +297,33 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_wait(bar(B_VFULL(j % ST)), (j / ST) & 1, &never, lim);
       }
     }
-  } else if (warp == kWarpMma) {
+   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && nt > 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, 0, 0);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, HD, 0, 1);
+      // descriptors of the operand bases; advancing along K adds (bytes >> 4) to the
+      // start-address field, which cannot carry out of its 14 bits for shared memory
+      const uint64_t dq0 = sdesc_sw128(sbase + OFF_Q, 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(sbase + OFF_K, 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(sbase + OFF_V, BOX, 1024);
       auto issue_qk = [&](int x, int st) {
+        const uint64_t ad = dq0 + (uint64_t)((x * TILE) >> 4);
+        const uint64_t bd = dk0 + (uint64_t)((st * TILE) >> 4);
+        const uint32_t d = tmem + TM_S + 128u * x;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint32_t off = (uint32_t)((kk >> 2) * BOX + (kk & 3) * 32);
-          const uint64_t ad = sdesc_sw128(sbase + OFF_Q + x * TILE + off, 16, 1024);
-          const uint64_t bd = sdesc_sw128(sbase + OFF_K + st * TILE + off, 16, 1024);
-          mma_ss(tmem + TM_S + 128u * x, ad, bd, idesc_qk, kk > 0 ? 1u : 0u);
+          const uint64_t off = (uint64_t)(((kk >> 2) * BOX + (kk & 3) * 32) >> 4);
+          mma_ss(d, ad + off, bd + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
       };
       auto issue_pv = [&](int x, int st, bool acc) {
+        const uint64_t bd = dv0 + (uint64_t)((st * TILE) >> 4);
+        const uint32_t d = tmem + TM_O + 128u * x;
+        const uint32_t pa = tmem + TM_S + 128u * x;
 #pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(sbase + OFF_V + st * TILE + kk * 2048, BOX, 1024);
-          mma_ts(tmem + TM_O + 128u * x, tmem + TM_S + 128u * x + 8u * kk, bd, idesc_pv, (acc || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < BN / 16; ++kk)
+          mma_ts(d, pa + 8u * kk, bd + (uint64_t)((kk * 2048) >> 4), idesc_pv, (acc || kk > 0) ? 1u : 0u);
       };
       bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_KFULL(0)), 0, abort_flag, T);
       if (!ok) fail(P, abort_flag, 3);
@@ -288,7 +371,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(bar(B_DRAIN()));
       mbar_wait(bar(B_DRAIN()), 0, &never, 100000000ull);
     }
+   }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsSoftmax));
     // ------------------------------------------------------------ softmax
     const int x = warp >> 2;          // query tile
     const int wq = warp & 3;          // TMEM lane quarter
@@ -300,26 +385,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tS = trow + TM_S + 128u * x;
     const uint32_t tO = trow + TM_O + 128u * x;
     float4* tab = reinterpret_cast<float4*>(smem + OFF_TAB) + x * 2 * BN;
+    // scores stay in raw units z = q.k (+ bias / scale); one FMA per element maps
+    // them to log2 units for the exponent: p = 2^(z * sc - m)
+    const float sc = P.scale_log2;
+    const float cb = P.coef_log2 / sc;
+    const uint64_t SC2 = pk2(sc, sc);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
+    // per-row correspondence of the (at most two) source frames of a tile,
+    // loaded one tile ahead so that the global-load latency overlaps a tile
+    Corr nxt = load_corr(a, tiles, 0, nt, p, row_ok, cb);
     for (int j = 0; j < nt; ++j) {
       const TileInfo ti = tiles[j];
-      float uxA = 0.f, uyA = 0.f, cA = 0.f, uxB = 0.f, uyB = 0.f, cB = 0.f;
+      const Corr cur = nxt;
+      nxt = load_corr(a, tiles, j + 1, nt, p, row_ok, cb);
       float4* tb = tab + (j & 1) * BN;
-      if (ti.cls == CLS_GENERAL) {
+      if (ti.cls != CLS_PLAIN) {
         const KeyInfo ki = key_info_of(a, ti.tile * BN + twg);
-        const float sel = ki.src < 0 ? 0.f : (ki.src == ti.sA ? 1.f : 2.f);
-        tb[twg] = make_float4(ki.x, ki.y, sel, ki.active ? 1.f : 0.f);
-        if (row_ok && ti.sA >= 0) {
-          const int64_t ia = (int64_t)p * a.S + ti.sA, ib = (int64_t)p * a.S + ti.sB;
-          if (a.valid[ia]) {
-            const float2 u = reinterpret_cast<const float2*>(a.uv)[ia];
-            uxA = u.x; uyA = u.y; cA = P.coef_log2;
-          }
-          if (a.valid[ib]) {
-            const float2 u = reinterpret_cast<const float2*>(a.uv)[ib];
-            uxB = u.x; uyB = u.y; cB = P.coef_log2;
-          }
+        if (ti.cls == CLS_BIAS1) {
+          reinterpret_cast<float2*>(tb)[twg] = make_float2(ki.x, ki.y);
+        } else {
+          const float sel = ki.src < 0 ? 0.f : (ki.src == ti.sA ? 1.f : 2.f);
+          tb[twg] = make_float4(ki.x, ki.y, sel, ki.active ? 1.f : 0.f);
         }
         named_bar_sync(1 + x, BM);
       }
@@ -329,55 +416,88 @@ __global__ void __launch_bounds__(kThreads, 1)
       // reach the same named barriers, so none of them can be left waiting
       if (!ok) continue;
       tc_fence_after();
-      uint32_t sr[4][32];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32u * c, sr[c]);
-      tmem_wait_ld();
-      float mt = -INFINITY;
-      if (ti.cls == CLS_PLAIN) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const float z = __uint_as_float(sr[c][e]) * P.scale_log2;
-            sr[c][e] = __float_as_uint(z);
-            mt = fmaxf(mt, z);
-          }
-      } else {
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
+      if (ti.cls == CLS_GENERAL) {
+        // rare tiles (segment or frame boundaries, masked keys): per-column bias and
+        // mask applied in place in TMEM, 32 columns at a time
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t g[32];
+          tmem_ld32(tS + 32u * c, g);
+          tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 32; ++e) {
             const float4 t = tb[32 * c + e];
             const bool selB = t.z > 1.5f;
-            const float ux = selB ? uxB : uxA, uy = selB ? uyB : uyA;
-            const float cf = t.z > 0.5f ? (selB ? cB : cA) : 0.f;
+            const float ux = selB ? cur.uxB : cur.uxA, uy = selB ? cur.uyB : cur.uyA;
+            const float cf = t.z > 0.5f ? (selB ? cur.cB : cur.cA) : 0.f;
             const float dx = t.x - ux, dy = t.y - uy;
-            float z = fmaf(cf, fmaf(dx, dx, dy * dy), __uint_as_float(sr[c][e]) * P.scale_log2);
-            z = t.w > 0.5f ? z : -INFINITY;
-            sr[c][e] = __float_as_uint(z);
-            mt = fmaxf(mt, z);
+            const float z = fmaf(cf, fmaf(dx, dx, dy * dy), __uint_as_float(g[e]));
+            g[e] = __float_as_uint(t.w > 0.5f ? z : -INFINITY);
           }
+          tmem_st32(tS + 32u * c, g);
+        }
+        tmem_wait_st();
       }
+      uint32_t sr[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32u * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
+      tmem_wait_ld();
+      if (ti.cls == CLS_BIAS1) {
+        // all 128 keys in one source frame: z += cA ((x - ux)^2 + (y - uy)^2), two columns per op
+        const uint64_t UX2 = pk2(cur.uxA, cur.uxA), UY2 = pk2(cur.uyA, cur.uyA), CA2 = pk2(cur.cA, cur.cA);
+        const float4* t4 = tb;
+#pragma unroll
+        for (int c = 0; c < 128; c += 2) {
+          const float4 t = t4[c >> 1];
+          const uint64_t dx = fsub2(pk2(t.x, t.z), UX2);
+          const uint64_t dy = fsub2(pk2(t.y, t.w), UY2);
+          const uint64_t d2 = ffma2(dy, dy, fmul2(dx, dx));
+          const uint64_t z = ffma2(d2, CA2, pk2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])));
+          float z0, z1;
+          upk2(z, z0, z1);
+          sr[c] = __float_as_uint(z0);
+          sr[c + 1] = __float_as_uint(z1);
+        }
+      }
+      // row max by a tree of three-input max operations
+      float mx[43];
+#pragma unroll
+      for (int i = 0; i < 42; ++i)
+        mx[i] = max3f(__uint_as_float(sr[3 * i]), __uint_as_float(sr[3 * i + 1]), __uint_as_float(sr[3 * i + 2]));
+      mx[42] = fmaxf(__uint_as_float(sr[126]), __uint_as_float(sr[127]));
+#pragma unroll
+      for (int i = 0; i < 14; ++i) mx[i] = max3f(mx[3 * i], mx[3 * i + 1], mx[3 * i + 2]);
+      mx[14] = mx[42];
+#pragma unroll
+      for (int i = 0; i < 5; ++i) mx[i] = max3f(mx[3 * i], mx[3 * i + 1], mx[3 * i + 2]);
+      const float mt = max3f(max3f(mx[0], mx[1], mx[2]), mx[3], mx[4]) * sc;
       // base-2 online softmax; the max is refreshed only when it grows by > 8
       const float mnew = fmaxf(m, mt);
       const bool resc = mnew > m + 8.f;
       const float factor = resc ? ex2(m - mnew) : 1.f;
       if (resc) m = mnew;
-      float rs = 0.f;
-      uint32_t pk[2][32];
+      const uint64_t NM2 = pk2(-m, -m);
+      uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
+      for (int half = 0; half < 2; ++half) {
+        uint32_t pk[32];
 #pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          const float p0 = ex2(__uint_as_float(sr[c][e]) - m);
-          const float p1 = ex2(__uint_as_float(sr[c][e + 1]) - m);
-          rs += p0 + p1;
-          pk[c >> 1][(c & 1) * 16 + e / 2] = pack_bf16x2(p0, p1);
+        for (int e = 0; e < 32; ++e) {
+          const int c = 64 * half + 2 * e;
+          const uint64_t t = ffma2(pk2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), SC2, NM2);
+          float t0, t1;
+          upk2(t, t0, t1);
+          const float p0 = ex2(t0), p1 = ex2(t1);
+          acc[e & 3] = fadd2(acc[e & 3], pk2(p0, p1));
+          pk[e] = pack_bf16x2(p0, p1);
         }
-      l = l * factor + rs;
-      tmem_st32(tS, pk[0]);
-      tmem_st32(tS + 32u, pk[1]);
+        tmem_st32(tS + 32u * half, pk);
+      }
+      float s0, s1, s2, s3;
+      upk2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), s0, s1);
+      (void)s2;
+      (void)s3;
+      l = l * factor + (s0 + s1);
       if (__any_sync(0xffffffffu, resc && j > 0)) {
         // PV of the previous tile has retired (it precedes this tile's S commit)
 #pragma unroll
