@@ -159,7 +159,9 @@ def algorithmic(W):
     # reprojection: query depth, per pair u^ (8 B) + cell (4 B) + flag (1 B) + source depth lookup (4 B)
     reproj = wl.Nq * 4 + wl.Nq * S * (8 + 4 + 1 + 4)
     update = 2 * wl.L * wl.Nc * row * 3 + wl.Nc * 4 * 2  # read new K/V, write slab + window; depth
-    return dict(flops=flops, gather_bytes=gather + score, reproj_bytes=reproj, update_bytes=update)
+    attn_bytes = wl.L * (2 * wl.Nq * row + 2 * act_keys * row)  # Q read, O written, K and V read
+    return dict(flops=flops, gather_bytes=gather + score, reproj_bytes=reproj, update_bytes=update,
+                attn_bytes=attn_bytes)
 
 
 def run_step(W, stream, ev=None):
@@ -187,6 +189,11 @@ def run_step(W, stream, ev=None):
 
 
 LAUNCHES_PER_STEP = 4
+
+# DRAM bytes (read + write) per layer of attn_tc_kernel at the Wan-1.3B chunk shape, from one
+# ncu capture of a 2-layer launch (283.4 MB / 2); traffic grows in proportion to layers.
+# Valid only for that shape and the kernel version it was captured on.
+ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.7e6}
 
 
 # ---------------------------------------------------------------------------- oracle arm
@@ -383,7 +390,10 @@ def main():
         "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel", "achieved": attn_tflops,
                      "peak": peaks["bf16_sus"], "unit": "TFLOP/s", "frac": attn_tflops / peaks["bf16_sus"],
                      "peak_source": f"{peaks['src']} bf16 sustained (kernel timed inside a long step)",
-                     "traffic": None},
+                     "frac_of_burst": attn_tflops / peaks["bf16"],
+                     "traffic": (ATTN_DRAM_BYTES_PER_LAYER[(wl.H, wl.Nq, wl.n_keys)] * wl.L
+                                 if (wl.H, wl.Nq, wl.n_keys) in ATTN_DRAM_BYTES_PER_LAYER else None),
+                     "traffic_algorithmic": alg["attn_bytes"]},
         "e2e": {"value": alg["flops"] * world / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h)},
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,

@@ -38,6 +38,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// try_wait that lets the hardware suspend the thread until the phase completes
+// (or `hint_ns` elapses), so that waiting warps do not spin on issue slots.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ uint64_t globaltimer() {
   uint64_t t;
   asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
@@ -45,13 +58,17 @@ __device__ __forceinline__ uint64_t globaltimer() {
 }
 
 // Bounded wait: gives up after `limit_ns` nanoseconds or once *abort is set, so
-// that no wait can spin forever.  Returns false on give-up.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort, uint64_t limit_ns) {
-  if (mbar_try_wait(bar, parity)) return true;
+// that no wait can spin forever.  Returns false on give-up.  With hint_ns = 0 the
+// thread polls; otherwise each try_wait may suspend it for up to hint_ns, which
+// frees issue slots for the other warps of its sub-partition.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort, uint64_t limit_ns,
+                                          uint32_t hint_ns = 0) {
+  auto attempt = [&]() { return hint_ns ? mbar_try_wait_sleep(bar, parity, hint_ns) : mbar_try_wait(bar, parity); };
+  if (attempt()) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 0) {
+    if (attempt()) return true;
+    if (hint_ns != 0 || (it & 255u) == 0) {
       if (*abort) return false;
       if (globaltimer() - t0 > limit_ns) return false;
     }
