@@ -2,17 +2,37 @@
 //
 //   A_pk = q_p . k_k / sqrt(d) + lambda B_s(p, k),  B = -||u_k - u^_s(p)||^2 / (2 sigma^2)
 //
-// on retrieved-slot key columns with a valid correspondence, 0 elsewhere; the
-// bias is evaluated per (query row, key column) inside the tile loop and never
-// written anywhere.  bf16 Q/K/V, fp32 scores, softmax and accumulation, bf16 O.
+// on retrieved-slot key columns with a valid correspondence, 0 elsewhere.  The
+// bias is never written to memory: the tensor core adds it to S.  KV tiles are cut
+// at every segment start and, inside retrieved segments, at every frame start, so
+// that each tile has at most one source frame; a tile's ragged tail is masked the
+// same way.  bf16 Q/K/V, fp32 scores, softmax and accumulation, bf16 O.
+//
+// Bias on the tensor core.  With coordinates relative to the frame centre
+// (x' = x - (w-1)/2, y' = y - (h-1)/2) and A = lambda log2(e) / (2 sigma^2) in base-2
+// units (0 when the pair is invalid), the bias of Eq. 2 expands as
+//   A (q_k - 2 ux' x'_k - 2 uy' y'_k + ux'^2 + uy'^2),   q_k = x'_k^2 + y'_k^2,
+// a dot product of a 4-vector per query row with a 4-vector per key.  Each query
+// coefficient is split into three bf16 terms (hi + mid + lo, ~24 bits) and q_k into
+// two (exact: x', y' are half-integers), giving a K = 16 extension of the QK^T
+// contraction whose products are exact in fp32:
+//   query row: [a0h a0h a0m a0m a0l a0l a1h a1m a1l a2h a2m a2l a3h a3m a3l 1]
+//   key row:   [qh  ql  qh  ql  qh  ql  x'  x'  x'  y'  y'  y'  1   1   1   M]
+// The last column masks keys past the tile's end (M = -2^100, else 0); an unbiased
+// tile has zeros in the first fifteen key columns.  One extra tcgen05.mma
+// (M = N = 128, K = 16, no-swizzle K-major operands) per query tile adds it to S,
+// and the softmax never touches individual columns.
 //
 // Structure (one CTA = two 128-row query tiles of one (layer, head)):
-//   warps 0-3  softmax of query tile 0   (TMEM lanes 0-127 of S0/O0)
-//   warps 4-7  softmax of query tile 1   (TMEM lanes 0-127 of S1/O1)
-//   warp  8    TMA producer: Q once, then K/V tiles of 128 keys, 2 stages each,
-//              128-byte swizzled boxes of 128 rows x 64 elements
-//   warp  9    TMEM owner and single-thread tcgen05.mma issuer
-//   warps 10-11 idle (they complete the third warpgroup for the register split)
+//   warps 0-3   softmax of query tile 0   (TMEM lanes 0-127 of S0/O0)
+//   warps 4-7   softmax of query tile 1   (TMEM lanes 0-127 of S1/O1)
+//   warp  8     TMA producer: Q once, then K/V tiles of 128 keys, 2 stages each,
+//               128-byte swizzled boxes of 128 rows x 64 elements
+//   warp  9     TMEM owner and single-thread tcgen05.mma issuer
+//   warps 10-11 build, ahead of use, the key-side bias/mask operand of every tile
+//               that needs one (3-deep ring, mbarrier handshake with the MMA warp)
+// The query-side bias operand of each query tile is written by its own softmax
+// warpgroup whenever the source frame of the next biased tile changes.
 // TMEM (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each.  S = Q K^T is an
 // SS MMA (both operands K-major in shared memory); each softmax thread reads its
 // row of S, writes P in bf16 over the first 64 columns of the same S buffer and
@@ -21,15 +41,15 @@
 // the tensor core works on one tile while the other tile's softmax runs.
 // Online softmax in base 2 with the row max kept stale until it grows by more
 // than 2^8 (exact: the same max normalises P, O and the row sum); O in TMEM is
-// rescaled only on those rare steps.  KV tiles that hold no active key (an empty
-// retrieved slot, keys past the cache end) are skipped by every role.
+// rescaled only on those rare steps.  Keys outside every segment and retrieved
+// slots without a chunk produce no tile at all.
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 #include <math.h>
 #include <string.h>
 
 #include "internal.cuh"
-#include "keys.cuh"
 #include "tc_ptx.cuh"
 
 namespace crc {
@@ -43,43 +63,53 @@ constexpr int BN = 128;  // keys per KV tile
 constexpr int HD = 128;  // head dim
 constexpr int NQT = 2;   // query tiles per CTA
 constexpr int ST = 2;    // stages for K and for V
-constexpr int kThreads = 384;  // 3 warpgroups: softmax 0, softmax 1, producer/MMA
+constexpr int kThreads = 384;  // 3 warpgroups: softmax 0, softmax 1, producer/MMA/tables
 constexpr int kWarpTma = 8;
 constexpr int kWarpMma = 9;
 // register split (setmaxnreg): the block launches with 384 x 168 registers; the
-// producer warpgroup drops to 96 and each softmax warpgroup rises to 200:
-// 2 x 128 x 200 + 128 x 96 <= 384 x 168.
+// producer warpgroup drops to 104 and each softmax warpgroup rises to 200:
+// 2 x 128 x 200 + 128 x 104 = 384 x 168.
 constexpr int kRegsSoftmax = 200;
-constexpr int kRegsProducer = 96;
+constexpr int kRegsProducer = 104;
 static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsProducer <= kThreads * 168, "register split exceeds the launch");
 constexpr int BOX = BM * 64 * 2;  // 128 rows x 64 bf16 = 16 KB
 constexpr int TILE = 2 * BOX;     // 128 rows x 128 bf16 = 32 KB
-constexpr int kMaxTiles = 1024;   // KV tiles per call
+constexpr int AUG = 128 * 16 * 2; // 128 rows x 16 bf16 bias operand = 4 KB
+constexpr int kMaxTiles = 640;    // KV tiles per call (keys <= 81920)
+constexpr int NBB = 3;            // ring of key-side bias/mask operands
+// mbarrier wait policy per role (0 = poll; otherwise the suspend hint in ns)
+constexpr uint32_t kHintSoftmax = 0;
+constexpr uint32_t kHintMma = 0;
+constexpr uint32_t kHintLoad = 0;
+constexpr uint32_t kHintTable = 0;
 
 constexpr int OFF_Q = 0;
 constexpr int OFF_K = OFF_Q + NQT * TILE;
 constexpr int OFF_V = OFF_K + ST * TILE;
-constexpr int OFF_TAB = OFF_V + ST * TILE;
-constexpr int TAB_BYTES = NQT * 2 * BN * 16;
-constexpr int OFF_TILES = OFF_TAB + TAB_BYTES;
-constexpr int OFF_BAR = OFF_TILES + kMaxTiles * 8;
-constexpr int NBAR = 1 + 4 * ST + 3 * NQT + 1;
+constexpr int OFF_AQ = OFF_V + ST * TILE;      // query-side bias operand, one per query tile
+constexpr int OFF_RB = OFF_AQ + NQT * AUG;     // key-side bias/mask operand ring
+constexpr int OFF_TILES = OFF_RB + NBB * AUG;
+constexpr int OFF_BAR = OFF_TILES + kMaxTiles * 12;
+constexpr int NBAR = 1 + 4 * ST + 3 * NQT + 1 + NQT + 2 * NBB;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
 constexpr int SMEM_BYTES = OFF_MISC + 64 + 1024;  // + slack for 1024-byte alignment
+static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 
 constexpr uint32_t TM_S = 0;    // S/P of tile x at column 128 x
 constexpr uint32_t TM_O = 256;  // O of tile x at column 256 + 128 x
 constexpr uint32_t TM_COLS = 512;
 
-constexpr uint8_t CLS_PLAIN = 0;    // every column active, none biased
-constexpr uint8_t CLS_BIAS1 = 1;    // every column active and biased, one source frame
-constexpr uint8_t CLS_GENERAL = 2;  // anything else: per-column bias / mask
+constexpr uint8_t CLS_PLAIN = 0;  // 128 active keys, no bias: Q K^T only
+constexpr uint8_t CLS_AUG = 1;    // biased and/or ragged: Q K^T + bias/mask operand
 
 struct TileInfo {
-  uint16_t tile;
+  uint32_t key0;    // first key of the tile
+  uint8_t nact_m1;  // active keys - 1 (keys key0 .. key0 + nact - 1)
   uint8_t cls;
-  int8_t sA, sB;  // the (at most two) source frames of biased columns, -1 if none
-  uint8_t pad[3];
+  int8_t s;         // source frame of the (biased) keys, -1 for an unbiased tile
+  uint8_t pad;
+  uint16_t q;       // ordinal among CLS_AUG tiles (ring position)
+  uint16_t loc0;    // index of key0 inside its source frame (biased tiles)
 };
 
 struct TcParams {
@@ -99,6 +129,9 @@ __device__ __forceinline__ int B_SFULL(int x) { return 1 + 4 * ST + x; }
 __device__ __forceinline__ int B_PREADY(int x) { return 1 + 4 * ST + NQT + x; }
 __device__ __forceinline__ int B_OFINAL(int x) { return 1 + 4 * ST + 2 * NQT + x; }
 __device__ __forceinline__ int B_DRAIN() { return 1 + 4 * ST + 3 * NQT; }
+__device__ __forceinline__ int B_AREADY(int x) { return 2 + 4 * ST + 3 * NQT + x; }
+__device__ __forceinline__ int B_BFULL(int b) { return 2 + 4 * ST + 4 * NQT + b; }
+__device__ __forceinline__ int B_BEMPTY(int b) { return 2 + 4 * ST + 4 * NQT + NBB + b; }
 
 // ---- packed fp32 pairs (Blackwell f32x2 ALU ops) and three-input max ----------
 __device__ __forceinline__ uint64_t pk2(float a, float b) {
@@ -119,49 +152,74 @@ __device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
-__device__ __forceinline__ uint64_t fsub2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
 __device__ __forceinline__ float max3f(float a, float b, float c) {
   float d;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
 }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t bf16_bits(float v) {
+  return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v));
+}
+// v ~= hi + mid + lo in bf16 (each term rounded to nearest from the remainder)
+__device__ __forceinline__ void split3(float v, uint32_t& h, uint32_t& m, uint32_t& l) {
+  const __nv_bfloat16 bh = __float2bfloat16_rn(v);
+  const float r1 = v - __bfloat162float(bh);
+  const __nv_bfloat16 bm = __float2bfloat16_rn(r1);
+  const float r2 = r1 - __bfloat162float(bm);
+  h = (uint32_t)__bfloat16_as_ushort(bh);
+  m = (uint32_t)__bfloat16_as_ushort(bm);
+  l = bf16_bits(r2);
+}
+// Write one 16-element bf16 row (given as 8 packed words) of a no-swizzle K-major
+// 128 x 16 operand: 8-row x 16-byte core matrices, K halves 128 bytes apart,
+// 8-row groups 256 bytes apart.
+__device__ __forceinline__ void store_aug_row(uint8_t* base, int row, const uint32_t (&w)[8]) {
+  uint8_t* p = base + (row >> 3) * 256 + (row & 7) * 16;
+  *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+  *reinterpret_cast<uint4*>(p + 128) = make_uint4(w[4], w[5], w[6], w[7]);
+}
 
 // One query row's correspondences in the two source frames of a KV tile, with the
 // bias coefficient already zero for invalid pairs (exact fallback).
 struct Corr {
-  float uxA, uyA, cA, uxB, uyB, cB;
+  float uxA, uyA, cA;
 };
 
 __device__ __forceinline__ Corr load_corr(const AttnArgs& a, const TileInfo* tiles, int j, int nt, int p, bool row_ok,
                                           float coef) {
-  Corr c{0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  Corr c{0.f, 0.f, 0.f};
   if (j >= nt || !row_ok) return c;
   const TileInfo ti = tiles[j];
-  if (ti.sA < 0) return c;
-  const int64_t ia = (int64_t)p * a.S + ti.sA, ib = (int64_t)p * a.S + ti.sB;
-  const float2* uv = reinterpret_cast<const float2*>(a.uv);
+  if (ti.s < 0) return c;
+  const int64_t ia = (int64_t)p * a.S + ti.s;
   if (__ldg(a.valid + ia)) {
-    const float2 u = __ldg(uv + ia);
+    const float2 u = __ldg(reinterpret_cast<const float2*>(a.uv) + ia);
     c.uxA = u.x;
     c.uyA = u.y;
     c.cA = coef;
   }
-  if (__ldg(a.valid + ib)) {
-    const float2 u = __ldg(uv + ib);
-    c.uxB = u.x;
-    c.uyB = u.y;
-    c.cB = coef;
-  }
   return c;
+}
+
+// Query-side bias operand row for source frame A of `c` (raw score units).
+__device__ __forceinline__ void aug_query_row(const Corr& c, float xc, float yc, float inv_sc, uint32_t (&w)[8]) {
+  const float A = c.cA * inv_sc;
+  const float ux = c.uxA - xc, uy = c.uyA - yc;
+  uint32_t a0[3], a1[3], a2[3], a3[3];
+  split3(A, a0[0], a0[1], a0[2]);
+  split3(-2.f * A * ux, a1[0], a1[1], a1[2]);
+  split3(-2.f * A * uy, a2[0], a2[1], a2[2]);
+  split3(A * fmaf(ux, ux, uy * uy), a3[0], a3[1], a3[2]);
+  w[0] = a0[0] | (a0[0] << 16);
+  w[1] = a0[1] | (a0[1] << 16);
+  w[2] = a0[2] | (a0[2] << 16);
+  w[3] = a1[0] | (a1[1] << 16);
+  w[4] = a1[2] | (a2[0] << 16);
+  w[5] = a2[1] | (a2[2] << 16);
+  w[6] = a3[0] | (a3[1] << 16);
+  w[7] = a3[2] | (bf16_bits(1.f) << 16);  // mask column
 }
 
 __device__ __forceinline__ void fail(const TcParams& P, volatile int* abort_flag, int code) {
@@ -186,6 +244,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + OFF_MISC + 4);
   int* ntiles_slot = reinterpret_cast<int*>(smem + OFF_MISC + 8);
   TileInfo* tiles = reinterpret_cast<TileInfo*>(smem + OFF_TILES);
+  const float xc = 0.5f * (float)(a.w - 1), yc = 0.5f * (float)(a.h - 1);
 
   if (tid == 0) {
     mbar_init(bar(B_QFULL()), 1);
@@ -199,51 +258,51 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(B_SFULL(x)), 1);
       mbar_init(bar(B_PREADY(x)), BM);
       mbar_init(bar(B_OFINAL(x)), 1);
+      mbar_init(bar(B_AREADY(x)), BM);
     }
     mbar_init(bar(B_DRAIN()), 1);
+    for (int b = 0; b < NBB; ++b) {
+      mbar_init(bar(B_BFULL(b)), 2);   // the two table warps
+      mbar_init(bar(B_BEMPTY(b)), 1);  // a tcgen05.commit after the tile's last MMA
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == 0) {
-    // compact list of KV tiles holding at least one active key, with their class
-    const int ntot = (a.Nk + BN - 1) / BN;
+    // KV tiles: each segment is cut into tiles of 128 keys from its start; retrieved
+    // segments are cut per source frame, so that a tile has at most one frame
     const int hw = a.h * a.w;
-    int count = 0;
-    for (int base = 0; base < ntot; base += 32) {
-      const int t = base + lane;
-      bool act = false;
-      TileInfo ti;
-      ti.tile = (uint16_t)t;
-      ti.cls = CLS_GENERAL;
-      ti.sA = -1;
-      ti.sB = -1;
-      if (t < ntot) {
-        const int k0 = t * BN, k1 = k0 + BN;
-        int nact = 0, nbias = 0, sA = 1 << 20, sB = -1;
-        for (int g = 0; g < a.nseg; ++g) {
-          const crc_segment sg = a.seg[g];
-          if (sg.length <= 0) continue;
-          const int lo = max(k0, sg.offset), hi = min(k1, sg.offset + sg.length);
-          if (lo >= hi) continue;
-          if (sg.kind == CRC_SEG_RETRIEVED) {
-            if (a.slot_chunk && a.slot_chunk[sg.slot] < 0) continue;
-            sA = min(sA, sg.slot * a.F + (lo - sg.offset) / hw);
-            sB = max(sB, sg.slot * a.F + (hi - 1 - sg.offset) / hw);
-            nbias += hi - lo;
-          }
-          nact += hi - lo;
+    int count = 0, qa = 0;
+    for (int g = 0; g < a.nseg; ++g) {
+      const crc_segment sg = a.seg[g];
+      if (sg.length <= 0) continue;
+      const bool ret = sg.kind == CRC_SEG_RETRIEVED;
+      if (ret && a.slot_chunk && a.slot_chunk[sg.slot] < 0) continue;  // empty slot: masked
+      const int nr = ret ? a.F : 1;
+      for (int rr = 0; rr < nr; ++rr) {
+        const int rstart = ret ? sg.offset + rr * hw : sg.offset;
+        const int rlen = ret ? hw : sg.length;
+        const int ntile = (rlen + BN - 1) / BN;
+        for (int base = 0; base < ntile; base += 32) {
+          const int t = base + lane;
+          const bool act = t < ntile;
+          TileInfo ti;
+          const int nact = act ? min(BN, rlen - t * BN) : 1;
+          ti.key0 = (uint32_t)(rstart + t * BN);
+          ti.nact_m1 = (uint8_t)(nact - 1);
+          ti.s = ret ? (int8_t)(sg.slot * a.F + rr) : (int8_t)-1;
+          ti.cls = (nact == BN && !ret) ? CLS_PLAIN : CLS_AUG;
+          ti.pad = 0;
+          ti.loc0 = (uint16_t)(t * BN);
+          const unsigned lt = (1u << lane) - 1u;
+          const unsigned m = __ballot_sync(0xffffffffu, act);
+          const unsigned ma = __ballot_sync(0xffffffffu, act && ti.cls == CLS_AUG);
+          ti.q = (uint16_t)(qa + __popc(ma & lt));
+          if (act) tiles[count + __popc(m & lt)] = ti;
+          count += __popc(m);
+          qa += __popc(ma);
         }
-        act = nact > 0;
-        if (sB >= 0) {
-          ti.sA = (int8_t)sA;
-          ti.sB = (int8_t)sB;
-        }
-        ti.cls = (nact == BN && sB < 0) ? CLS_PLAIN
-                 : (nact == BN && nbias == BN && sA == sB) ? CLS_BIAS1 : CLS_GENERAL;
       }
-      const unsigned m = __ballot_sync(0xffffffffu, act);
-      if (act) tiles[count + __popc(m & ((1u << lane) - 1u))] = ti;
-      count += __popc(m);
     }
     if (lane == 0) *ntiles_slot = count;
   }
@@ -274,13 +333,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < nt; ++j) {
         const int st = j % ST;
         const uint32_t par = ((j / ST) & 1) ^ 1;
-        const int key0 = tiles[j].tile * BN;
-        if (!mbar_wait(bar(B_KEMPTY(st)), par, abort_flag, T)) { fail(P, abort_flag, 1); break; }
+        const int key0 = (int)tiles[j].key0;
+        if (!mbar_wait(bar(B_KEMPTY(st)), par, abort_flag, T, kHintLoad)) { fail(P, abort_flag, 1); break; }
         mbar_arrive_expect_tx(bar(B_KFULL(st)), TILE);
         for (int b = 0; b < 2; ++b)
           tma_load_4d(sbase + OFF_K + st * TILE + b * BOX, &tmK, bar(B_KFULL(st)), b * 64, head, key0, layer);
         issued_k = j + 1;
-        if (!mbar_wait(bar(B_VEMPTY(st)), par, abort_flag, T)) { fail(P, abort_flag, 2); break; }
+        if (!mbar_wait(bar(B_VEMPTY(st)), par, abort_flag, T, kHintLoad)) { fail(P, abort_flag, 2); break; }
         mbar_arrive_expect_tx(bar(B_VFULL(st)), TILE);
         for (int b = 0; b < 2; ++b)
           tma_load_4d(sbase + OFF_V + st * TILE + b * BOX, &tmV, bar(B_VFULL(st)), b * 64, head, key0, layer);
@@ -297,6 +356,50 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_wait(bar(B_VFULL(j % ST)), (j / ST) & 1, &never, lim);
       }
     }
+   } else if (warp > kWarpMma) {
+    // ------------------------------------------------------------ tables
+    // Warps 10-11 (64 threads, two keys each) build the key-side bias/mask operand
+    // of every CLS_AUG tile ahead of the MMA warp.
+    const int bt = tid - (kWarpMma + 1) * 32;
+    const uint32_t one = bf16_bits(1.f), neg = bf16_bits(-0x1p100f);
+    for (int j = 0; j < nt; ++j) {
+      const TileInfo ti = tiles[j];
+      if (ti.cls != CLS_AUG) continue;
+      const int b = ti.q % NBB;
+      if (!mbar_wait(bar(B_BEMPTY(b)), ((ti.q / NBB) & 1) ^ 1, abort_flag, T, kHintTable)) {
+        fail(P, abort_flag, 9);
+        break;
+      }
+      uint8_t* blk = smem + OFF_RB + b * AUG;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int row = 2 * bt + h;
+        const uint32_t mask = row <= (int)ti.nact_m1 ? 0u : neg;
+        uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, mask << 16};
+        if (ti.s >= 0) {
+          // grid cell of the key inside its source frame, relative to the frame centre
+          const int loc = (int)ti.loc0 + row;
+          const int yi = loc / a.w;
+          const float xr = (float)(loc - yi * a.w) - xc, yr = (float)yi - yc;
+          const float q = fmaf(xr, xr, yr * yr);
+          const uint32_t qh = bf16_bits(q);
+          const uint32_t ql = bf16_bits(q - __bfloat162float(__ushort_as_bfloat16((unsigned short)qh)));
+          const uint32_t xb = bf16_bits(xr), yb = bf16_bits(yr);
+          w[0] = qh | (ql << 16);
+          w[1] = w[0];
+          w[2] = w[0];
+          w[3] = xb | (xb << 16);
+          w[4] = xb | (yb << 16);
+          w[5] = yb | (yb << 16);
+          w[6] = one | (one << 16);
+          w[7] = one | (mask << 16);
+        }
+        store_aug_row(blk, row, w);
+      }
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(B_BFULL(b)));
+    }
    } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && nt > 0) {
@@ -307,7 +410,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t dq0 = sdesc_sw128(sbase + OFF_Q, 16, 1024);
       const uint64_t dk0 = sdesc_sw128(sbase + OFF_K, 16, 1024);
       const uint64_t dv0 = sdesc_sw128(sbase + OFF_V, BOX, 1024);
-      auto issue_qk = [&](int x, int st) {
+      const uint64_t daq0 = sdesc_none(sbase + OFF_AQ, 128, 256);
+      const uint64_t dbk0 = sdesc_none(sbase + OFF_RB, 128, 256);
+      auto issue_qk = [&](int x, int st, const TileInfo& ti) {
         const uint64_t ad = dq0 + (uint64_t)((x * TILE) >> 4);
         const uint64_t bd = dk0 + (uint64_t)((st * TILE) >> 4);
         const uint32_t d = tmem + TM_S + 128u * x;
@@ -316,6 +421,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t off = (uint64_t)(((kk >> 2) * BOX + (kk & 3) * 32) >> 4);
           mma_ss(d, ad + off, bd + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
+        if (ti.cls == CLS_AUG)  // + bias/mask: query-side x key-side operand, K = 16
+          mma_ss(d, daq0 + (uint64_t)((x * AUG) >> 4), dbk0 + (uint64_t)(((ti.q % NBB) * AUG) >> 4), idesc_qk, 1u);
       };
       auto issue_pv = [&](int x, int st, bool acc) {
         const uint64_t bd = dv0 + (uint64_t)((st * TILE) >> 4);
@@ -325,42 +432,53 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < BN / 16; ++kk)
           mma_ts(d, pa + 8u * kk, bd + (uint64_t)((kk * 2048) >> 4), idesc_pv, (acc || kk > 0) ? 1u : 0u);
       };
-      bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_KFULL(0)), 0, abort_flag, T);
+      // wait until the key-side bias operand of tile ti is built
+      auto bias_ready = [&](const TileInfo& ti) {
+        return ti.cls != CLS_AUG ||
+               mbar_wait(bar(B_BFULL(ti.q % NBB)), (ti.q / NBB) & 1, abort_flag, T, kHintMma);
+      };
+      TileInfo t0 = tiles[0];
+      bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_KFULL(0)), 0, abort_flag, T) &&
+                mbar_wait(bar(B_AREADY(0)), 0, abort_flag, T) && mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T) &&
+                bias_ready(t0);
       if (!ok) fail(P, abort_flag, 3);
       if (ok) {
         tc_fence_after();
-        issue_qk(0, 0);
+        issue_qk(0, 0, t0);
         mma_commit(bar(B_SFULL(0)));
-        issue_qk(1, 0);
+        issue_qk(1, 0, t0);
         mma_commit(bar(B_SFULL(1)));
         mma_commit(bar(B_KEMPTY(0)));
+        if (t0.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(t0.q % NBB)));
         for (int j = 0; j < nt && ok; ++j) {
           const int st = j % ST;
           const int jn = j + 1, stn = jn % ST;
           const bool more = jn < nt;
-          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T) &&
-               mbar_wait(bar(B_VFULL(st)), (j / ST) & 1, abort_flag, T);
+          const TileInfo tn = more ? tiles[jn] : t0;
+          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma) &&
+               mbar_wait(bar(B_VFULL(st)), (j / ST) & 1, abort_flag, T, kHintMma);
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
           issue_pv(0, st, j > 0);
           if (more) {
-            ok = mbar_wait(bar(B_KFULL(stn)), (jn / ST) & 1, abort_flag, T);
+            ok = mbar_wait(bar(B_KFULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma) && bias_ready(tn);
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
-            issue_qk(0, stn);
+            issue_qk(0, stn, tn);
             mma_commit(bar(B_SFULL(0)));
           } else {
             mma_commit(bar(B_OFINAL(0)));
           }
-          ok = mbar_wait(bar(B_PREADY(1)), j & 1, abort_flag, T);
+          ok = mbar_wait(bar(B_PREADY(1)), j & 1, abort_flag, T, kHintMma);
           if (!ok) { fail(P, abort_flag, 6); break; }
           tc_fence_after();
           issue_pv(1, st, j > 0);
           mma_commit(bar(B_VEMPTY(st)));
           if (more) {
-            issue_qk(1, stn);
+            issue_qk(1, stn, tn);
             mma_commit(bar(B_SFULL(1)));
             mma_commit(bar(B_KEMPTY(stn)));
+            if (tn.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(tn.q % NBB)));
           } else {
             mma_commit(bar(B_OFINAL(1)));
           }
@@ -379,86 +497,40 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int wq = warp & 3;          // TMEM lane quarter
     const int r = wq * 32 + lane;     // row in tile = TMEM lane
     const int p = q0 + x * BM + r;    // query index
-    const int twg = tid - x * BM;     // thread index in the warpgroup
     const bool row_ok = p < a.Nq;
     const uint32_t trow = tmem + ((uint32_t)(wq * 32) << 16);
     const uint32_t tS = trow + TM_S + 128u * x;
     const uint32_t tO = trow + TM_O + 128u * x;
-    float4* tab = reinterpret_cast<float4*>(smem + OFF_TAB) + x * 2 * BN;
-    // scores stay in raw units z = q.k (+ bias / scale); one FMA per element maps
+    uint8_t* aq = smem + OFF_AQ + x * AUG;
+    // scores are in raw units z = q.k (+ bias / scale); one FMA per element maps
     // them to log2 units for the exponent: p = 2^(z * sc - m)
     const float sc = P.scale_log2;
-    const float cb = P.coef_log2 / sc;
+    const float inv_sc = 1.f / sc;
     const uint64_t SC2 = pk2(sc, sc);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     // per-row correspondence of the (at most two) source frames of a tile,
     // loaded one tile ahead so that the global-load latency overlaps a tile
-    Corr nxt = load_corr(a, tiles, 0, nt, p, row_ok, cb);
+    Corr nxt = load_corr(a, tiles, 0, nt, p, row_ok, P.coef_log2);
+    // query-side bias/mask operand: the first tile's source frame (or no bias)
+    int aug_frame = nt > 0 ? tiles[0].s : -1;
+    {
+      uint32_t w[8];
+      aug_query_row(nxt, xc, yc, inv_sc, w);
+      store_aug_row(aq, r, w);
+      fence_async_smem();
+    }
+    mbar_arrive(bar(B_AREADY(x)));
     for (int j = 0; j < nt; ++j) {
-      const TileInfo ti = tiles[j];
-      const Corr cur = nxt;
-      nxt = load_corr(a, tiles, j + 1, nt, p, row_ok, cb);
-      float4* tb = tab + (j & 1) * BN;
-      if (ti.cls != CLS_PLAIN) {
-        const KeyInfo ki = key_info_of(a, ti.tile * BN + twg);
-        if (ti.cls == CLS_BIAS1) {
-          reinterpret_cast<float2*>(tb)[twg] = make_float2(ki.x, ki.y);
-        } else {
-          const float sel = ki.src < 0 ? 0.f : (ki.src == ti.sA ? 1.f : 2.f);
-          tb[twg] = make_float4(ki.x, ki.y, sel, ki.active ? 1.f : 0.f);
-        }
-        named_bar_sync(1 + x, BM);
-      }
-      if (ok && !mbar_wait(bar(B_SFULL(x)), j & 1, abort_flag, T)) { fail(P, abort_flag, 7); ok = false; }
+      nxt = load_corr(a, tiles, j + 1, nt, p, row_ok, P.coef_log2);
+      if (ok && !mbar_wait(bar(B_SFULL(x)), j & 1, abort_flag, T, kHintSoftmax)) { fail(P, abort_flag, 7); ok = false; }
       ok = __all_sync(0xffffffffu, ok);
-      // after a failure keep walking the tile list: every warp of the group must
-      // reach the same named barriers, so none of them can be left waiting
-      if (!ok) continue;
+      if (!ok) break;
       tc_fence_after();
-      if (ti.cls == CLS_GENERAL) {
-        // rare tiles (segment or frame boundaries, masked keys): per-column bias and
-        // mask applied in place in TMEM, 32 columns at a time
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t g[32];
-          tmem_ld32(tS + 32u * c, g);
-          tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const float4 t = tb[32 * c + e];
-            const bool selB = t.z > 1.5f;
-            const float ux = selB ? cur.uxB : cur.uxA, uy = selB ? cur.uyB : cur.uyA;
-            const float cf = t.z > 0.5f ? (selB ? cur.cB : cur.cA) : 0.f;
-            const float dx = t.x - ux, dy = t.y - uy;
-            const float z = fmaf(cf, fmaf(dx, dx, dy * dy), __uint_as_float(g[e]));
-            g[e] = __float_as_uint(t.w > 0.5f ? z : -INFINITY);
-          }
-          tmem_st32(tS + 32u * c, g);
-        }
-        tmem_wait_st();
-      }
       uint32_t sr[128];
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32u * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
       tmem_wait_ld();
-      if (ti.cls == CLS_BIAS1) {
-        // all 128 keys in one source frame: z += cA ((x - ux)^2 + (y - uy)^2), two columns per op
-        const uint64_t UX2 = pk2(cur.uxA, cur.uxA), UY2 = pk2(cur.uyA, cur.uyA), CA2 = pk2(cur.cA, cur.cA);
-        const float4* t4 = tb;
-#pragma unroll
-        for (int c = 0; c < 128; c += 2) {
-          const float4 t = t4[c >> 1];
-          const uint64_t dx = fsub2(pk2(t.x, t.z), UX2);
-          const uint64_t dy = fsub2(pk2(t.y, t.w), UY2);
-          const uint64_t d2 = ffma2(dy, dy, fmul2(dx, dx));
-          const uint64_t z = ffma2(d2, CA2, pk2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])));
-          float z0, z1;
-          upk2(z, z0, z1);
-          sr[c] = __float_as_uint(z0);
-          sr[c + 1] = __float_as_uint(z1);
-        }
-      }
       // row max by a tree of three-input max operations
       float mx[43];
 #pragma unroll
@@ -493,10 +565,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st32(tS + 32u * half, pk);
       }
-      float s0, s1, s2, s3;
+      float s0, s1;
       upk2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), s0, s1);
-      (void)s2;
-      (void)s3;
       l = l * factor + (s0 + s1);
       if (__any_sync(0xffffffffu, resc && j > 0)) {
         // PV of the previous tile has retired (it precedes this tile's S commit)
@@ -508,6 +578,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
           tmem_st32(tO + 32u * c, o);
+        }
+      }
+      // the next tile's QK^T is issued only after this tile's P is ready, and this
+      // tile's QK^T has retired: the query-side bias operand can be rewritten here
+      if (j + 1 < nt) {
+        const TileInfo tn = tiles[j + 1];
+        if (tn.cls == CLS_AUG && tn.s >= 0 && tn.s != aug_frame) {
+          uint32_t w[8];
+          aug_query_row(nxt, xc, yc, inv_sc, w);
+          store_aug_row(aq, r, w);
+          fence_async_smem();
+          aug_frame = tn.s;
         }
       }
       tmem_wait_st();
@@ -583,10 +665,16 @@ bool make_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void*
 
 cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
   if (a.dtype != CRC_BF16 || a.d != HD) return cudaErrorNotSupported;
-  const int64_t ntiles = (a.Nk + BN - 1) / BN;
-  if (ntiles > kMaxTiles || a.S > 127) return cudaErrorNotSupported;
-  for (int g = 0; g < a.nseg; ++g)  // at most two source frames per KV tile
-    if (a.seg[g].kind == CRC_SEG_RETRIEVED && a.seg[g].length > 0 && a.h * a.w < BN) return cudaErrorNotSupported;
+  int64_t ntiles = 0;  // the kernel's tiling: per segment, per frame for retrieved segments
+  for (int g = 0; g < a.nseg; ++g) {
+    const crc_segment& sg = a.seg[g];
+    if (sg.length <= 0) continue;
+    if (sg.kind == CRC_SEG_RETRIEVED)
+      ntiles += (int64_t)a.F * ((a.h * a.w + BN - 1) / BN);
+    else
+      ntiles += (sg.length + BN - 1) / BN;
+  }
+  if (ntiles > kMaxTiles || a.S > 127 || a.h * a.w > 65535) return cudaErrorNotSupported;
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
   if (!al16(a.q) || !al16(a.k) || !al16(a.v) || !al16(a.o)) return cudaErrorNotSupported;
   const int64_t strides[9] = {a.q_sl, a.q_st, a.q_sh, a.k_sl, a.k_st, a.k_sh, a.o_sl, a.o_st, a.o_sh};

@@ -113,6 +113,16 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo_byt
   d |= (uint64_t)2 << 61;  // SWIZZLE_128B
   return d;
 }
+// Shared-memory matrix descriptor, no swizzle: 8-row x 16-byte core matrices;
+// lbo = byte distance between core matrices along K, sbo = along M/N.
+__device__ __forceinline__ uint64_t sdesc_none(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo_bytes & 0x3FFFFu) >> 4) << 16;
+  d |= (uint64_t)((sbo_bytes & 0x3FFFFu) >> 4) << 32;
+  d |= (uint64_t)1 << 46;  // descriptor version for tcgen05
+  return d;                // layout type 0: SWIZZLE_NONE
+}
 // Instruction descriptor for .kind::f16 with bf16 A/B and fp32 D.
 // a_mn / b_mn: operand is MN-major (1) instead of K-major (0).
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, int a_mn, int b_mn) {
