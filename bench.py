@@ -196,6 +196,182 @@ LAUNCHES_PER_STEP = 4
 ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.6e6}
 
 
+# ---------------------------------------------------------------------------- ranks
+def rank_seed(rank: int) -> int:
+    """Each rank draws its own synthetic Q/K/V (independent chunk streams)."""
+    return 1234 + rank
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The slowest rank's time: the whole job ends when the last rank ends."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_tflops(flops_per_rank_step: float, step_s: float, world: int) -> float:
+    """Weak scaling: every rank runs the same per-rank work; value = all ranks' FLOP / max time."""
+    return flops_per_rank_step * world / step_s / 1e12
+
+
+# ---------------------------------------------------------------------------- end to end
+E2E_INPUTS = ("q", "k_new", "v_new", "depth")
+
+
+def run_e2e(W, stream, steps: int):
+    """The step through the public API with host buffers, pipelined on two copy streams.
+
+    Every step copies its inputs (Q, the new chunk's K/V, its depth) from pinned host
+    memory and copies O back.  Two device buffer sets let step i+1's upload and step
+    i-1's download overlap step i's kernels.  Returns (seconds per step, h2d, d2h bytes)."""
+    import torch
+
+    host_in = {k: W[k].cpu().pin_memory() for k in E2E_INPUTS}
+    dev = [W, dict(W, **{k: torch.empty_like(W[k]) for k in E2E_INPUTS + ("o",)})]
+    host_out = [torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True) for _ in range(2)]
+    h2d_s, d2h_s = torch.cuda.Stream(), torch.cuda.Stream()
+    in_ready = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    out_read = [torch.cuda.Event() for _ in range(2)]
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    h2d_s.wait_stream(stream)
+    d2h_s.wait_stream(stream)
+
+    def upload(i):
+        b = i % 2
+        with torch.cuda.stream(h2d_s):
+            if i >= 2:
+                h2d_s.wait_event(done[b])  # step i-2 has finished reading buffer b
+            for k in E2E_INPUTS:
+                dev[b][k].copy_(host_in[k], non_blocking=True)
+            in_ready[b].record(h2d_s)
+
+    upload(0)
+    for i in range(steps):
+        b = i % 2
+        if i + 1 < steps:
+            upload(i + 1)
+        stream.wait_event(in_ready[b])
+        if i >= 2:
+            stream.wait_event(out_read[b])  # O of step i-2 has left buffer b
+        run_step(dev[b], stream)
+        done[b].record(stream)
+        with torch.cuda.stream(d2h_s):
+            d2h_s.wait_event(done[b])
+            host_out[b].copy_(dev[b]["o"], non_blocking=True)
+            out_read[b].record(d2h_s)
+    stream.wait_stream(h2d_s)
+    stream.wait_stream(d2h_s)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + W["frames"].nbytes
+    d2h = host_out[0].numel() * host_out[0].element_size()
+    return e0.elapsed_time(e1) / 1e3 / steps, h2d, d2h
+
+
+# ---------------------------------------------------------------------------- context
+def run_graph(W, steps: int):
+    """The same step captured once in a CUDA graph and replayed (launch overhead removed)."""
+    import torch
+
+    g = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        run_step(W, side)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g):
+        run_step(W, torch.cuda.current_stream())
+    g.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / 1e3 / steps
+
+
+def _bias_matrix(W):
+    """lambda * B of Eq. 2 as a dense [N_q, N_k] matrix, for the materialised-bias comparator."""
+    import torch
+
+    wl = W["wl"]
+    dev = W["q"].device
+    Bm = torch.zeros(wl.Nq, wl.n_keys, device=dev)
+    count = int(W["count"].item())
+    idx = W["idx"].tolist()
+    hw = wl.h * wl.w
+    for off, length, kind, slot in wl.segments:
+        if kind != 1 or length == 0 or slot >= count or idx[slot] < 0:
+            continue
+        local = torch.arange(length, device=dev)
+        s = slot * wl.F + local // hw
+        pix = local % hw
+        xk, yk = (pix % wl.w).float(), (pix // wl.w).float()
+        d2 = (xk - W["uv"][:, s, 0]) ** 2 + (yk - W["uv"][:, s, 1]) ** 2
+        b = -wl.lam * d2 / (2.0 * wl.sigma ** 2)
+        Bm[:, off:off + length] = torch.where(W["valid"][:, s].bool(), b, torch.zeros_like(b))
+    return Bm.to(W["q"].dtype)
+
+
+def sdpa_context(W, flops: float, iters: int = 5):
+    """PyTorch SDPA on the same tensors: plain attention (lambda = 0) and attention with
+    the bias materialised as an additive mask.  Context only, not the measured path."""
+    import torch
+    import torch.nn.functional as Fn
+    from torch.nn.attention import SDPBackend, sdpa_kernel
+
+    q = W["q"].permute(0, 2, 1, 3)
+    k = W["cache"].k.permute(0, 2, 1, 3)
+    v = W["cache"].v.permute(0, 2, 1, 3)
+    out = {}
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(iters):
+            r = fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / 1e3 / iters, r
+
+    backends = [("cudnn", SDPBackend.CUDNN_ATTENTION), ("flash", SDPBackend.FLASH_ATTENTION),
+                ("efficient", SDPBackend.EFFICIENT_ATTENTION)]
+    mask = None
+    for label, use_bias in (("lambda0", False), ("materialised_bias", True)):
+        if use_bias:
+            mask = _bias_matrix(W)[None, None].expand(q.shape[0], q.shape[1], -1, -1)
+        for name, be in backends:
+            try:
+                with sdpa_kernel([be]):
+                    t, r = timed(lambda: Fn.scaled_dot_product_attention(q, k, v, attn_mask=mask))
+            except RuntimeError as exc:
+                out.setdefault(label, {})[name] = f"unavailable: {str(exc).splitlines()[0][:80]}"
+                continue
+            entry = {"ms": t * 1e3, "tflops": flops / t / 1e12}
+            if use_bias:
+                entry["max_abs_diff_vs_crc"] = float((r.permute(0, 2, 1, 3).float() - W["o"].float()).abs().max())
+            out.setdefault(label, {})[name] = entry
+    if mask is not None:
+        out["materialised_bias"]["mask_bytes"] = int(mask.shape[2] * mask.shape[3] * mask.element_size())
+    return out
+
+
 # ---------------------------------------------------------------------------- oracle arm
 def oracle_sample(cfg_id: int, layers: int, budget_s: float):
     """Time the fp64 oracle on a bounded sample of one step: the full retrieval and
@@ -294,6 +470,7 @@ def main():
     ap.add_argument("--layers", type=int, default=30)
     ap.add_argument("--impl", default="crc", choices=["crc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-context", action="store_true", help="skip the PyTorch SDPA comparators")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
@@ -314,7 +491,7 @@ def main():
     from paper_2607_21848_gb300 import build
 
     build.build()
-    W = setup(args.config, args.layers, device, seed=1234 + rank)
+    W = setup(args.config, args.layers, device, seed=rank_seed(rank))
     wl = W["wl"]
     alg = algorithmic(W)
     stream = torch.cuda.current_stream()
@@ -337,39 +514,18 @@ def main():
             run_step(W, stream, evs[i])
         t_end.record(stream)
         barrier()
-    elapsed = t_start.elapsed_time(t_end) / 1e3
+    elapsed = max_over_ranks(t_start.elapsed_time(t_end) / 1e3, world, device)
     assert W["status"].item() == 0, "attention kernel reported a pipeline timeout"
-    if world > 1:
-        t = torch.tensor([elapsed], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
     stage = {nm: statistics.median(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(args.steps)) / 1e3
              for j, nm in enumerate(["update", "retrieve", "correspond", "attention"])}
     step_s = elapsed / args.steps
-    value = alg["flops"] * world / step_s / 1e12
+    value = whole_job_tflops(alg["flops"], step_s, world)
 
-    # end to end through the public API with host buffers: pinned inputs in, output out
-    host_in = {k: W[k].cpu().pin_memory() for k in ("q", "k_new", "v_new", "depth")}
-    host_out = torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True)
-    h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + W["frames"].nbytes
-    d2h = host_out.numel() * host_out.element_size()
-    e2e_steps = max(3, min(args.steps, 20))
     barrier()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(e2e_steps):
-        for k, t in host_in.items():
-            W[k].copy_(t, non_blocking=True)
-        run_step(W, stream)
-        host_out.copy_(W["o"], non_blocking=True)
-    e1.record(stream)
-    barrier()
-    e2e_s = e0.elapsed_time(e1) / 1e3 / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_s], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s, h2d, d2h = run_e2e(W, stream, max(3, min(args.steps, 20)))
+    e2e_s = max_over_ranks(e2e_s, world, device)
+    graph_s = run_graph(W, max(3, min(args.steps, 20)))
+    context = sdpa_context(W, alg["flops"]) if not args.no_context else None
 
     peaks = _peaks()
     attn_tflops = alg["flops"] / stage["attention"] / 1e12
@@ -394,11 +550,16 @@ def main():
                      "traffic": (ATTN_DRAM_BYTES_PER_LAYER[(wl.H, wl.Nq, wl.n_keys)] * wl.L
                                  if (wl.H, wl.Nq, wl.n_keys) in ATTN_DRAM_BYTES_PER_LAYER else None),
                      "traffic_algorithmic": alg["attn_bytes"]},
-        "e2e": {"value": alg["flops"] * world / e2e_s / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": int(h2d),
-                "d2h_bytes_per_step": int(d2h)},
+        "e2e": {"value": whole_job_tflops(alg["flops"], e2e_s, world), "unit": "TFLOP/s",
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
+                "pipelining": "two device buffer sets; uploads and downloads on two copy streams overlap the kernels"},
+        "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
+                  "note": "one step captured in a CUDA graph and replayed"},
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,
         "clocks": clk.summary(),
     }
+    if context is not None:
+        line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path"}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cb = oracle_sample(args.config, args.layers, 10.0)
         line["cpu_baseline"] = {

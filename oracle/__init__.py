@@ -13,6 +13,8 @@ from .crc_oracle import (  # noqa: F401
     gather,
     key_table,
     reproject,
+    rope_frequencies,
+    rope_reposition,
     retrieval_terms,
     retrieve,
 )

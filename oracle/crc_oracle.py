@@ -13,6 +13,7 @@ Training-Free Revisit Consistency for Autoregressive Generative Rendering"):
   retrieve          Sec. 4.2, Eq. 1 (score s(j), admissible set A_n, empty-set fallback)
   fill_slots        Sec. 4.2 (an empty A_n makes the retrieved slot extend the recent window)
   gather            Sec. 4.2 (retrieved chunk reinstated into the clean cache)
+  rope_reposition   Sec. 4.2 "Cache packing" (re-packed chunk moved to positions next to the window)
   reproject         Sec. 4.3, Eq. 3 (reprojection warp)
   correspond        Sec. 4.3, Eq. 3-4 and the design choices (visibility test, exact fallback)
   key_table         Sec. 4.3 design choice (ii) (which key columns carry a bias)
@@ -84,9 +85,11 @@ def retrieval_terms(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n
 
 
 def retrieve(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n: np.ndarray, n: int,
-             E: float, w_v: float, tau_c: float, cos_tau_v: float, delta: int, k: int):
+             E: float, w_v: float, tau_c: float, cos_tau_v: float, delta: int, k: int,
+             exclude_sink: bool = False):
     """Eq. 1: score every historical chunk j, keep the admissible set A_n, and return
-    the k admissible chunks closest in pose (ascending (s, j)).
+    the k admissible chunks closest in pose (ascending (s, j)).  With exclude_sink
+    the anchor chunk j = 0 (always in the cache already) is never admissible.
 
     Returns (idx [k] int32 padded with -1, score [k] fp64 padded with +inf, count).
     """
@@ -94,6 +97,8 @@ def retrieve(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n: np.nd
     s, dist, dot = retrieval_terms(bank_c, bank_v, c_n, v_n, E, w_v)
     j = np.arange(B)
     adm = (dist <= tau_c) & (dot >= cos_tau_v) & ((n - j) >= delta)
+    if exclude_sink:
+        adm &= j != 0
     cand = sorted((float(s[i]), int(i)) for i in np.nonzero(adm)[0])
     count = min(k, len(cand))
     idx = np.full(k, -1, dtype=np.int32)
@@ -115,9 +120,51 @@ def fill_slots(idx: np.ndarray, count: int, ext_first: int, ext_min: int) -> np.
     return out
 
 
-def gather(pool: np.ndarray, slot_chunks: np.ndarray, num_slabs: int) -> List[Optional[np.ndarray]]:
-    """Reinstate chunk slot_chunks[r] (slab chunk % num_slabs of pool [P, 2, L, Nc, H, d])."""
-    return [None if j < 0 else pool[j % num_slabs] for j in slot_chunks]
+def rope_frequencies(pairs: int, theta: float) -> np.ndarray:
+    """Angular frequency of each temporal rotary pair i: theta^(-i / pairs)."""
+    return np.array([theta ** (-(i / pairs)) for i in range(pairs)], dtype=np.float64)
+
+
+def rope_reposition(x: np.ndarray, delta: float, channel0: int, pairs: int, theta: float,
+                    interleaved: bool) -> np.ndarray:
+    """Sec. 4.2 "Cache packing": move keys that carry a rotary embedding at temporal
+    position t to position t + delta.  Each temporal pair (x_a, x_b) is read as the
+    complex number x_a + i x_b and multiplied by exp(i delta omega_i).  Pair i sits at
+    channels (channel0 + 2i, channel0 + 2i + 1) when interleaved, else at
+    (channel0 + i, channel0 + i + pairs).  x [..., d] is widened to fp64."""
+    out = np.array(x, dtype=np.float64)
+    omega = rope_frequencies(pairs, theta)
+    for i in range(pairs):
+        if interleaved:
+            a, b = channel0 + 2 * i, channel0 + 2 * i + 1
+        else:
+            a, b = channel0 + i, channel0 + i + pairs
+        z = (out[..., a] + 1j * out[..., b]) * np.exp(1j * (delta * omega[i]))
+        out[..., a] = z.real
+        out[..., b] = z.imag
+    return out
+
+
+def gather(pool: np.ndarray, slot_chunks: np.ndarray, num_slabs: int,
+           rope: Optional[dict] = None) -> List[Optional[np.ndarray]]:
+    """Reinstate chunk slot_chunks[r] (slab chunk % num_slabs of pool [P, 2, L, Nc, H, d]).
+
+    With `rope` (keys channel0, pairs, theta, interleaved, pos_slot0, pos_stride,
+    frame_pos0, F) the keys of slot r, cached at positions frame_pos0 + j F + f, are
+    moved to pos_slot0 + r pos_stride + f (Sec. 4.2 "Cache packing": the retrieved
+    chunk is re-packed next to the recent window).  Values carry no rotary embedding."""
+    out: List[Optional[np.ndarray]] = []
+    for r, j in enumerate(slot_chunks):
+        if j < 0:
+            out.append(None)
+            continue
+        slab = np.array(pool[j % num_slabs], dtype=np.float64)
+        if rope is not None and rope["pairs"] > 0:
+            delta = (rope["pos_slot0"] + r * rope["pos_stride"]) - (rope["frame_pos0"] + int(j) * rope["F"])
+            slab[0] = rope_reposition(slab[0], delta, rope["channel0"], rope["pairs"], rope["theta"],
+                                      rope["interleaved"])
+        out.append(slab)
+    return out
 
 
 # ----------------------------------------------------------------------------

@@ -98,6 +98,17 @@ def test_retrieval_gates_flip_at_threshold():
     assert s[0] == 0.5 + 0.5
 
 
+def test_exclude_sink_removes_only_the_anchor_chunk():
+    # chunk 0 is the best match; chunk 2 the second best (Sec. 4.2: the anchor is always in the cache)
+    bc = np.array([[0.1, 0.0, 0.0], [5.0, 0.0, 0.0], [0.2, 0.0, 0.0]])
+    bv = np.tile([1.0, 0.0, 0.0], (3, 1))
+    args = (np.zeros(3), np.array([1.0, 0.0, 0.0]), 10, 1.0, 0.5, math.inf, -1.0, 1, 2)
+    idx, _, count = oracle.retrieve(bc, bv, *args)
+    assert count == 2 and list(idx) == [0, 2]
+    idx, _, count = oracle.retrieve(bc, bv, *args, exclude_sink=True)
+    assert count == 2 and list(idx) == [2, 1]
+
+
 def test_retrieval_ties_break_by_chunk_index():
     bc = np.array([[1.0, 0, 0], [0, 1.0, 0], [1.0, 0, 0], [0, 0, 1.0]])
     bv = np.tile([1.0, 0.0, 0.0], (4, 1))
@@ -481,3 +492,95 @@ def test_source_frame_index_spans_slots():
     assert blk.argmax() == 1 * w + 1 and blk.max() == pytest.approx(W[0, 0, 0, 0], rel=1e-14)
     # slot 0 and the first frame of slot 1 are not biased for query 0
     np.testing.assert_allclose(W[0, 0, 0, Nc:2 * Nc + h * w], W[0, 0, 0, 0], rtol=1e-14)
+
+
+# ----------------------------------------------------------------------------
+# RoPE re-positioning of a re-packed chunk (Sec. 4.2 "Cache packing")
+# ----------------------------------------------------------------------------
+
+
+def _rotary(x, pos, channel0, pairs, theta, interleaved):
+    """Standard rotary embedding written with explicit 2x2 rotation matrices: pair i of
+    a token at position pos is rotated by the angle pos * theta^(-i/pairs)."""
+    out = np.array(x, dtype=np.float64)
+    pos = np.asarray(pos, dtype=np.float64)
+    for i in range(pairs):
+        a, b = (channel0 + 2 * i, channel0 + 2 * i + 1) if interleaved else (channel0 + i, channel0 + i + pairs)
+        ang = pos * theta ** (-i / pairs)
+        ca, sa = np.cos(ang), np.sin(ang)
+        xa, xb = out[..., a].copy(), out[..., b].copy()
+        out[..., a] = ca * xa - sa * xb
+        out[..., b] = sa * xa + ca * xb
+    return out
+
+
+def test_rope_handworked_quarter_turn_and_frequency():
+    # pair 0 has frequency 1: a shift of 1 rotates (1, 0) by one radian, counter-clockwise
+    x = np.array([1.0, 0.0, 0.3, 0.7])
+    y = oracle.rope_reposition(x, 1, 0, 2, 4.0 / math.pi ** 2, True)
+    assert abs(y[0] - 0.5403023058681398) < 1e-15 and abs(y[1] - 0.8414709848078965) < 1e-15
+    # pair 1 has frequency theta^(-1/2) = pi/2 for theta = 4/pi^2: a quarter turn (a, b) -> (-b, a)
+    assert abs(y[2] + 0.7) < 1e-15 and abs(y[3] - 0.3) < 1e-15
+    # half-split layout: pair 0 = channels (0, 2), pair 1 = channels (1, 3)
+    z = oracle.rope_reposition(np.array([1.0, 0.3, 0.0, 0.7]), 1, 0, 2, 4.0 / math.pi ** 2, False)
+    assert abs(z[0] - 0.5403023058681398) < 1e-15 and abs(z[2] - 0.8414709848078965) < 1e-15
+    assert abs(z[1] + 0.7) < 1e-15 and abs(z[3] - 0.3) < 1e-15
+
+
+@pytest.mark.parametrize("interleaved", [True, False])
+def test_rope_reposition_equals_embedding_at_new_position(interleaved):
+    g = np.random.default_rng(3)
+    d, c0, pairs, theta = 32, 8, 8, 10000.0
+    k = g.normal(size=(5, d))
+    q = g.normal(size=(5, d))
+    for t, delta in ((7, 5), (40, -33), (3, 0)):
+        moved = oracle.rope_reposition(_rotary(k, t, c0, pairs, theta, interleaved), delta, c0, pairs, theta,
+                                       interleaved)
+        np.testing.assert_allclose(moved, _rotary(k, t + delta, c0, pairs, theta, interleaved), atol=1e-12)
+        # relative positions: moving the key by delta equals moving the query by -delta
+        m = 11
+        lhs = np.sum(_rotary(q, m, c0, pairs, theta, interleaved) * moved, axis=-1)
+        rhs = np.sum(_rotary(q, m - delta, c0, pairs, theta, interleaved) * _rotary(k, t, c0, pairs, theta,
+                                                                                   interleaved), axis=-1)
+        np.testing.assert_allclose(lhs, rhs, atol=1e-12)
+        # channels outside the temporal block are untouched; pair norms are kept
+        outside = np.r_[0:c0, c0 + 2 * pairs:d]
+        np.testing.assert_array_equal(moved[:, outside], k[:, outside])
+        np.testing.assert_allclose(np.linalg.norm(moved, axis=-1), np.linalg.norm(k, axis=-1), rtol=1e-14)
+
+
+def test_rope_reposition_composes_and_half_split_is_a_channel_permutation():
+    g = np.random.default_rng(4)
+    x = g.normal(size=(3, 16))
+    a = oracle.rope_reposition(oracle.rope_reposition(x, 4, 0, 6, 500.0, True), -9, 0, 6, 500.0, True)
+    np.testing.assert_allclose(a, oracle.rope_reposition(x, -5, 0, 6, 500.0, True), atol=1e-13)
+    # half-split pair i = (c0 + i, c0 + i + pairs) is interleaved pair i after moving the channels
+    c0, pairs = 2, 6
+    perm = np.arange(16)
+    perm[c0:c0 + 2 * pairs:2] = np.arange(c0, c0 + pairs)
+    perm[c0 + 1:c0 + 2 * pairs:2] = np.arange(c0 + pairs, c0 + 2 * pairs)
+    half = oracle.rope_reposition(x, 7, c0, pairs, 300.0, False)
+    inter = oracle.rope_reposition(x[:, perm], 7, c0, pairs, 300.0, True)
+    np.testing.assert_allclose(half[:, perm], inter, atol=1e-13)
+
+
+def test_gather_repositions_keys_next_to_the_window():
+    # keys cached with their rotary embedding at frame positions frame_pos0 + j F + f; after the
+    # gather, slot r's frame f sits at pos_slot0 + r pos_stride + f.  Values are not rotated.
+    g = np.random.default_rng(5)
+    F, h, w, L, H, d, P = 2, 2, 3, 2, 2, 16, 4
+    Nc = F * h * w
+    frame = np.repeat(np.arange(F), h * w)[None, :, None]
+    rope = dict(channel0=0, pairs=8, theta=10000.0, interleaved=True, pos_slot0=30, pos_stride=F, frame_pos0=-2,
+                F=F)
+    raw = g.normal(size=(P, 2, L, Nc, H, d))
+    pool = raw.copy()
+    chunks = [9, 6]  # chunk j lives in slab j % P
+    for j in chunks:
+        pool[j % P, 0] = _rotary(raw[j % P, 0], rope["frame_pos0"] + j * F + frame, 0, 8, 1e4, True)
+    out = oracle.gather(pool, np.array(chunks + [-1]), P, rope=rope)
+    for r, j in enumerate(chunks):
+        want = _rotary(raw[j % P, 0], rope["pos_slot0"] + r * F + frame, 0, 8, 1e4, True)
+        np.testing.assert_allclose(out[r][0], want, atol=1e-12)
+        np.testing.assert_array_equal(out[r][1], pool[j % P, 1])
+    assert out[2] is None
