@@ -63,6 +63,7 @@ typedef int32_t crc_status;
 #define CRC_MAX_SEGMENTS 16
 #define CRC_MAX_FRAMES 4   /* frames per chunk, F */
 #define CRC_MAX_K 8        /* retrieved slots per step, k */
+#define CRC_MAX_ROPE_PAIRS 64  /* temporal rotary pairs per head, crc_rope.pairs */
 
 /* One latent frame's camera annotation (Sec. 4.1): intrinsics K rescaled to the
  * token grid, camera-to-world rotation R and camera centre c, all row-major fp64.
@@ -139,7 +140,36 @@ typedef struct {
   int32_t ext_first; /* fallback: slot r >= count holds chunk ext_first-(r-count)  */
   int32_t ext_min;   /*   if that is >= ext_min (else the slot stays empty);       */
                      /*   ext_first < 0 disables the fallback                      */
+  int32_t exclude_sink; /* non-zero: chunk 0 (the anchor, always cached) is never  */
+                        /*   admissible; 0 keeps the literal reading of Eq. 1      */
 } crc_retrieval;
+
+/* RoPE re-positioning of re-packed chunks (Sec. 4.2 "Cache packing": a retrieved
+ * chunk is re-packed at rotary positions adjacent to the recent window).
+ *
+ * Keys are cached after their rotary embedding, at the temporal position of the
+ * latent frame that produced them: frame f of chunk j sits at
+ * frame_pos0 + j*F + f.  Gathered into retrieved slot r, that frame is moved to
+ * pos_slot0 + r*pos_stride + f, i.e. every temporal rotary pair i of every head is
+ * multiplied, as the complex number k[a] + i k[b], by exp(i delta_r omega_i) with
+ *   omega_i = theta^(-i / pairs),  delta_r = pos_slot0 + r*pos_stride - frame_pos0 - j*F.
+ * Pair i occupies channels (channel0 + 2i, channel0 + 2i + 1) of the head when
+ * `interleaved`, else (channel0 + i, channel0 + i + pairs).  Only the temporal
+ * block is rotated (the spatial rotary axes of a chunk do not move) and values
+ * carry no rotary embedding.  The rotation runs in fp32 with fp64 angles and is
+ * rounded once to the cache dtype.  pairs = 0 (or a NULL crc_rope) copies the
+ * keys unchanged.  Layout limits: channel0 + 2*pairs <= d, pairs <= 64; with
+ * `interleaved` channel0 is even; without it channel0 and pairs are multiples of
+ * 16 bytes' worth of elements (8 for bf16, 4 for fp32). */
+typedef struct {
+  int32_t channel0;
+  int32_t pairs;
+  int32_t interleaved;
+  int32_t pos_slot0;
+  int32_t pos_stride;
+  int32_t frame_pos0;
+  double theta;
+} crc_rope;
 
 /* ---- library information ------------------------------------------------- */
 const char* crc_version(void);
@@ -197,12 +227,33 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
  *   d_count [1] int32: number of admissible chunks retrieved (<= k).
  * Then, for every CRC_SEG_RETRIEVED segment of `cache` with slot r < k and
  * d_idx[r] >= 0, keys [offset, offset+N_c) of every layer receive the K and V
- * of slab d_idx[r] % num_slabs (the gather).  Everything stays on the device.
+ * of slab d_idx[r] % num_slabs (the gather), the keys re-positioned by `rope`
+ * when it is not NULL.  Everything stays on the device.
  * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE, CRC_ERR_UNSUPPORTED, CRC_ERR_CUDA.
  */
 crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
-                        int32_t n, const crc_retrieval* p, const crc_cache* cache, int32_t* d_idx, double* d_score,
-                        int32_t* d_count, cudaStream_t s);
+                        int32_t n, const crc_retrieval* p, const crc_cache* cache, const crc_rope* rope,
+                        int32_t* d_idx, double* d_score, int32_t* d_count, cudaStream_t s);
+
+/*
+ * crc_gather — the gather half of crc_retrieve for a second cache that mirrors
+ * the main one (Sec. 4.2 "Cache packing": the retrieved chunk is reinstated in
+ * the control-branch cache too; that branch takes no correspondence bias).
+ *
+ *   pool      device [num_slabs][2][L][N_c][H][d] K (0) / V (1) slabs, dense, dtype
+ *             of the call; chunk j lives in slab j % num_slabs.  The shape's L and
+ *             H are those of the mirrored cache (e.g. the control blocks only).
+ *   d_idx     device [k] int32 chunk of each retrieved slot, as written by
+ *             crc_retrieve (negative = empty slot, left untouched).
+ *   cache     every CRC_SEG_RETRIEVED segment with slot r < k and length N_c
+ *             receives slab d_idx[r] % num_slabs; other keys are not touched.
+ *   rope      NULL, or the re-positioning of the keys as for crc_retrieve.
+ * Errors: CRC_ERR_INVALID_ARG (null pointers, k out of 1..CRC_MAX_K, bad rope),
+ * CRC_ERR_SHAPE (cache strides, two segments for one slot), CRC_ERR_UNSUPPORTED
+ * (alignment, rope layout), CRC_ERR_CUDA.
+ */
+crc_status crc_gather(const crc_shape* shape, const void* pool, int32_t num_slabs, const int32_t* d_idx, int32_t k,
+                      const crc_cache* cache, const crc_rope* rope, cudaStream_t s);
 
 /*
  * crc_correspond — Sec. 4.3, Eq. 3-4.  For every query token p = (t, i, j) of

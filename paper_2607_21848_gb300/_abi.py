@@ -28,6 +28,7 @@ CRC_SEG_WINDOW = 2
 CRC_MAX_SEGMENTS = 16
 CRC_MAX_FRAMES = 4
 CRC_MAX_K = 8
+CRC_MAX_ROPE_PAIRS = 64
 
 CRC_ATTN_DEFAULT = 0
 CRC_ATTN_SIMT = 1
@@ -63,7 +64,13 @@ class crc_bank(C.Structure):
 
 class crc_retrieval(C.Structure):
     _fields_ = [("E", C.c_double), ("w_v", C.c_double), ("tau_c", C.c_double), ("cos_tau_v", C.c_double),
-                ("delta", C.c_int32), ("k", C.c_int32), ("ext_first", C.c_int32), ("ext_min", C.c_int32)]
+                ("delta", C.c_int32), ("k", C.c_int32), ("ext_first", C.c_int32), ("ext_min", C.c_int32),
+                ("exclude_sink", C.c_int32)]
+
+
+class crc_rope(C.Structure):
+    _fields_ = [("channel0", C.c_int32), ("pairs", C.c_int32), ("interleaved", C.c_int32), ("pos_slot0", C.c_int32),
+                ("pos_stride", C.c_int32), ("frame_pos0", C.c_int32), ("theta", C.c_double)]
 
 
 _P = C.POINTER
@@ -76,7 +83,10 @@ _SIGS = {
     "crc_cache_update": (C.c_int32, [_P(crc_bank), _P(crc_shape), C.c_int32, _P(crc_frame), C.c_void_p, C.c_void_p,
                                      C.c_void_p, _P(crc_cache), C.c_int32, C.c_void_p]),
     "crc_retrieve": (C.c_int32, [_P(crc_bank), C.c_int32, _P(crc_shape), _P(crc_frame), C.c_int32,
-                                 _P(crc_retrieval), _P(crc_cache), C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+                                 _P(crc_retrieval), _P(crc_cache), _P(crc_rope), C.c_void_p, C.c_void_p, C.c_void_p,
+                                 C.c_void_p]),
+    "crc_gather": (C.c_int32, [_P(crc_shape), C.c_void_p, C.c_int32, C.c_void_p, C.c_int32, _P(crc_cache),
+                               _P(crc_rope), C.c_void_p]),
     "crc_correspond": (C.c_int32, [_P(crc_shape), _P(crc_frame), C.c_void_p, _P(crc_bank), C.c_void_p, C.c_void_p,
                                    C.c_int32, C.c_float, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "crc_biased_attention": (C.c_int32, [_P(crc_shape), crc_tensor, _P(crc_cache), crc_tensor, C.c_void_p, C.c_int32,

@@ -115,8 +115,14 @@ class Cache:
 
 
 def retrieval_params(E: float, w_v: float, tau_c: float, cos_tau_v: float, delta: int, k: int,
-                     ext_first: int = -1, ext_min: int = 0) -> _abi.crc_retrieval:
-    return _abi.crc_retrieval(E, w_v, tau_c, cos_tau_v, delta, k, ext_first, ext_min)
+                     ext_first: int = -1, ext_min: int = 0, exclude_sink: bool = False) -> _abi.crc_retrieval:
+    return _abi.crc_retrieval(E, w_v, tau_c, cos_tau_v, delta, k, ext_first, ext_min, int(bool(exclude_sink)))
+
+
+def rope_params(channel0: int, pairs: int, theta: float, interleaved: bool, pos_slot0: int, pos_stride: int,
+                frame_pos0: int = 0) -> _abi.crc_rope:
+    """Temporal RoPE re-positioning of gathered keys (crc_rope in include/crc.h)."""
+    return _abi.crc_rope(channel0, pairs, int(bool(interleaved)), pos_slot0, pos_stride, frame_pos0, float(theta))
 
 
 def crc_version() -> str:
@@ -146,15 +152,28 @@ def crc_cache_update(bank: Bank, shp: _abi.crc_shape, chunk: int, frames: np.nda
 
 def crc_retrieve(bank: Bank, bank_count: int, shp: _abi.crc_shape, cur_frames: np.ndarray, n: int,
                  params: _abi.crc_retrieval, cache: Optional[Cache], idx: torch.Tensor, score: Optional[torch.Tensor],
-                 count: torch.Tensor, stream=None) -> None:
+                 count: torch.Tensor, stream=None, rope: Optional[_abi.crc_rope] = None) -> None:
     lib = _abi.load()
     fr = frames_struct(cur_frames)
     b = bank.struct()
     cs = cache.struct() if cache is not None else None
     _abi.check("crc_retrieve",
                lib.crc_retrieve(C.byref(b), bank_count, C.byref(shp), fr, n, C.byref(params),
-                                C.byref(cs) if cs is not None else None, _ptr(idx), _ptr(score), _ptr(count),
-                                _stream(stream)))
+                                C.byref(cs) if cs is not None else None, C.byref(rope) if rope is not None else None,
+                                _ptr(idx), _ptr(score), _ptr(count), _stream(stream)))
+
+
+def crc_gather(shp: _abi.crc_shape, pool: torch.Tensor, idx: torch.Tensor, k: int, cache: Cache,
+               rope: Optional[_abi.crc_rope] = None, stream=None) -> None:
+    """Mirror the retrieved slots d_idx of a step into a second cache from its own slab pool
+    `pool` [num_slabs, 2, L, N_c, H, d]."""
+    lib = _abi.load()
+    if pool.dim() != 6 or not pool.is_contiguous():
+        raise ValueError("expected a dense [num_slabs, 2, L, N_c, H, d] slab pool")
+    cs = cache.struct()
+    _abi.check("crc_gather",
+               lib.crc_gather(C.byref(shp), _ptr(pool), pool.shape[0], _ptr(idx), k, C.byref(cs),
+                              C.byref(rope) if rope is not None else None, _stream(stream)))
 
 
 def crc_correspond(shp: _abi.crc_shape, cur_frames: np.ndarray, depth: torch.Tensor, bank: Bank, idx: torch.Tensor,

@@ -77,6 +77,65 @@ crc_status check_cache(const crc_cache* c, const crc_shape* sh) {
   return CRC_OK;
 }
 
+// RoPE layout limits of crc_rope (see include/crc.h).
+crc_status check_rope(const crc_rope* r, const crc_shape* sh) {
+  if (!r || r->pairs == 0) return CRC_OK;
+  if (r->pairs < 0 || r->pairs > CRC_MAX_ROPE_PAIRS || r->channel0 < 0 || !(r->theta > 0.0) || !isfinite(r->theta) ||
+      (r->interleaved != 0 && r->interleaved != 1))
+    return CRC_ERR_INVALID_ARG;
+  if ((int64_t)r->channel0 + 2LL * r->pairs > sh->d) return CRC_ERR_INVALID_ARG;
+  const int epv = 16 / elem_bytes(sh->dtype);  // elements per 16-byte vector
+  if (r->interleaved ? (r->channel0 % 2 != 0) : (r->channel0 % epv != 0 || r->pairs % epv != 0))
+    return CRC_ERR_UNSUPPORTED;
+  return CRC_OK;
+}
+
+// Gather arguments for the retrieved segments of `cache` from a slab pool.
+crc_status fill_gather(crc::GatherArgs& g, const crc_shape* sh, const void* pool, int32_t num_slabs,
+                       const crc_cache* cache, int32_t k, const crc_rope* rope) {
+  crc_status st = check_cache(cache, sh);
+  if (st) return st;
+  if ((st = check_rope(rope, sh))) return st;
+  if (!pool || num_slabs < 1) return CRC_ERR_INVALID_ARG;
+  if (!aligned16(pool)) return CRC_ERR_UNSUPPORTED;
+  const int es = elem_bytes(sh->dtype);
+  const int32_t nc = sh->F * sh->h * sh->w;
+  const int32_t row_bytes = sh->H * sh->d * es;
+  g.pool = static_cast<const char*>(pool);
+  g.num_slabs = num_slabs;
+  g.kv_bytes = (int64_t)sh->L * nc * row_bytes;
+  g.slab_bytes = 2 * g.kv_bytes;
+  g.cache_k = static_cast<char*>(cache->k.data);
+  g.cache_v = static_cast<char*>(cache->v.data);
+  g.cache_layer_stride = cache->k.stride_layer * es;
+  g.cache_token_stride = cache->k.stride_token * es;
+  g.L = sh->L;
+  g.Nc = nc;
+  g.row_bytes = row_bytes;
+  g.d = sh->d;
+  g.elem_bytes = es;
+  g.F = sh->F;
+  for (int r = 0; r < CRC_MAX_K; ++r) g.slot_offset[r] = -1;
+  for (int i = 0; i < cache->nseg; ++i) {
+    const crc_segment& sg = cache->seg[i];
+    if (sg.kind == CRC_SEG_RETRIEVED && sg.slot < k && sg.length == nc) {
+      if (g.slot_offset[sg.slot] >= 0) return CRC_ERR_SHAPE;  // two segments for one slot
+      g.slot_offset[sg.slot] = sg.offset;
+    }
+  }
+  g.rope_pairs = 0;
+  if (rope && rope->pairs > 0) {
+    g.rope_pairs = rope->pairs;
+    g.rope_c0 = rope->channel0;
+    g.rope_interleaved = rope->interleaved;
+    g.rope_pos_slot0 = rope->pos_slot0;
+    g.rope_pos_stride = rope->pos_stride;
+    g.rope_frame_pos0 = rope->frame_pos0;
+    for (int i = 0; i < rope->pairs; ++i) g.rope_omega[i] = pow(rope->theta, -((double)i / (double)rope->pairs));
+  }
+  return CRC_OK;
+}
+
 void pack_frames(crc::FrameSet& fs, const crc_frame* fr, int F) {
   memset(&fs, 0, sizeof(fs));
   fs.F = F;
@@ -174,8 +233,8 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
 }
 
 crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
-                        int32_t n, const crc_retrieval* p, const crc_cache* cache, int32_t* d_idx, double* d_score,
-                        int32_t* d_count, cudaStream_t s) {
+                        int32_t n, const crc_retrieval* p, const crc_cache* cache, const crc_rope* rope,
+                        int32_t* d_idx, double* d_score, int32_t* d_count, cudaStream_t s) {
   crc_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_bank(bank, cache != nullptr))) return st;
@@ -199,37 +258,28 @@ crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shap
   a.k = p->k;
   a.ext_first = p->ext_first;
   a.ext_min = p->ext_min;
+  a.exclude_sink = p->exclude_sink != 0;
   a.d_idx = d_idx;
   a.d_score = d_score;
   a.d_count = d_count;
-  for (int r = 0; r < CRC_MAX_K; ++r) a.slot_offset[r] = -1;
-  if (cache) {
-    if ((st = check_cache(cache, shape))) return st;
-    const int es = elem_bytes(shape->dtype);
-    const int32_t nc = shape->F * shape->h * shape->w;
-    const int32_t row_bytes = shape->H * shape->d * es;
-    if (!aligned16(bank->kv)) return CRC_ERR_UNSUPPORTED;
-    a.pool = static_cast<const char*>(bank->kv);
-    a.num_slabs = bank->num_slabs;
-    a.layer_bytes = (int64_t)nc * row_bytes;
-    a.kv_bytes = (int64_t)shape->L * a.layer_bytes;
-    a.slab_bytes = 2 * a.kv_bytes;
-    a.cache_k = static_cast<char*>(cache->k.data);
-    a.cache_v = static_cast<char*>(cache->v.data);
-    a.cache_layer_stride = cache->k.stride_layer * es;
-    a.cache_token_stride = cache->k.stride_token * es;
-    a.L = shape->L;
-    a.Nc = nc;
-    a.row_bytes = row_bytes;
-    for (int g = 0; g < cache->nseg; ++g) {
-      const crc_segment& sg = cache->seg[g];
-      if (sg.kind == CRC_SEG_RETRIEVED && sg.slot < p->k && sg.length == nc) {
-        if (a.slot_offset[sg.slot] >= 0) return CRC_ERR_SHAPE;  // two segments for one slot
-        a.slot_offset[sg.slot] = sg.offset;
-      }
-    }
-  }
+  if ((st = check_rope(rope, shape))) return st;
+  a.g.pool = nullptr;
+  if (cache && (st = fill_gather(a.g, shape, bank->kv, bank->num_slabs, cache, p->k, rope))) return st;
   cudaError_t e = crc::launch_retrieve(a, s);
+  return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+crc_status crc_gather(const crc_shape* shape, const void* pool, int32_t num_slabs, const int32_t* d_idx, int32_t k,
+                      const crc_cache* cache, const crc_rope* rope, cudaStream_t s) {
+  crc_status st = check_shape(shape);
+  if (st) return st;
+  if (!d_idx || !cache || k < 1 || k > CRC_MAX_K) return CRC_ERR_INVALID_ARG;
+  crc::GatherOnlyArgs a;
+  memset(&a, 0, sizeof(a));
+  a.d_idx = d_idx;
+  a.k = k;
+  if ((st = fill_gather(a.g, shape, pool, num_slabs, cache, k, rope))) return st;
+  cudaError_t e = crc::launch_gather(a, s);
   return e == cudaSuccess ? CRC_OK : cuda_fail(e);
 }
 

@@ -1,0 +1,193 @@
+// Gather of retrieved chunks from the slab pool into a cache (Sec. 4.2), with the
+// optional temporal RoPE re-positioning of the keys (Sec. 4.2 "Cache packing").
+//
+// Shared by the fused retrieval launch and the standalone mirror gather, so both
+// produce bit-identical cache contents for the same slots.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "copy.cuh"
+#include "internal.cuh"
+
+namespace crc {
+
+// Per-CTA plan of one gather: the chunk held by every slot, whether its keys are
+// rotated, and the (cos, sin) of each slot's rotation for every temporal pair.
+struct GatherPlan {
+  int32_t chunk[CRC_MAX_K];
+  int32_t rotate[CRC_MAX_K];
+  float2 cs[CRC_MAX_K][CRC_MAX_ROPE_PAIRS];
+};
+
+// Position shift of slot r holding chunk j: from frame_pos0 + j*F to pos_slot0 + r*pos_stride.
+__device__ __forceinline__ int64_t rope_delta(const GatherArgs& g, int r, int64_t j) {
+  return (int64_t)g.rope_pos_slot0 + (int64_t)r * g.rope_pos_stride - ((int64_t)g.rope_frame_pos0 + j * g.F);
+}
+
+// Fills plan.rotate[] and plan.cs[] once plan.chunk[] is visible to the whole block.
+// Angles are formed in fp64 (delta * omega_i) so that large position shifts keep
+// their accuracy; the rotation itself runs in fp32.  Ends with a block barrier.
+__device__ inline void plan_rope(const GatherArgs& g, int k, GatherPlan& p) {
+  for (int r = threadIdx.x; r < k; r += blockDim.x) {
+    const int64_t j = p.chunk[r];
+    p.rotate[r] = (g.rope_pairs > 0 && j >= 0 && rope_delta(g, r, j) != 0) ? 1 : 0;
+  }
+  const int n = k * g.rope_pairs;
+  for (int e = threadIdx.x; e < n; e += blockDim.x) {
+    const int r = e / g.rope_pairs, i = e - r * g.rope_pairs;
+    const int64_t j = p.chunk[r];
+    if (j < 0) continue;
+    double sn, cn;
+    sincos((double)rope_delta(g, r, j) * g.rope_omega[i], &sn, &cn);
+    p.cs[r][i] = make_float2((float)cn, (float)sn);
+  }
+  __syncthreads();
+}
+
+// (a + i b) * (cos + i sin), each product rounded separately.
+__device__ __forceinline__ void rotate_pair(float& a, float& b, float2 cs) {
+  const float na = __fsub_rn(__fmul_rn(a, cs.x), __fmul_rn(b, cs.y));
+  const float nb = __fadd_rn(__fmul_rn(a, cs.y), __fmul_rn(b, cs.x));
+  a = na;
+  b = nb;
+}
+
+// 16-byte vectors of the cache dtype widened to fp32 and rounded back (nearest even).
+template <bool BF16>
+struct Vec16;
+
+template <>
+struct Vec16<true> {
+  static constexpr int N = 8;
+  __device__ static __forceinline__ void unpack(const uint4& v, float x[8]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      x[2 * i] = __uint_as_float(w[i] << 16);
+      x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+  }
+  __device__ static __forceinline__ uint4 pack(const float x[8]) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 h = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
+      w[i] = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+  }
+};
+
+template <>
+struct Vec16<false> {
+  static constexpr int N = 4;
+  __device__ static __forceinline__ void unpack(const uint4& v, float x[4]) {
+    x[0] = __uint_as_float(v.x);
+    x[1] = __uint_as_float(v.y);
+    x[2] = __uint_as_float(v.z);
+    x[3] = __uint_as_float(v.w);
+  }
+  __device__ static __forceinline__ uint4 pack(const float x[4]) {
+    return make_uint4(__float_as_uint(x[0]), __float_as_uint(x[1]), __float_as_uint(x[2]), __float_as_uint(x[3]));
+  }
+};
+
+// One key row (H heads of d channels) copied by a warp with the temporal pairs of
+// every head rotated by cs[i].  Interleaved pairs lie inside one 16-byte vector
+// (channel0 is even).  Half-split pairs (c, c + pairs) lie in two vectors `half`
+// apart (channel0 and pairs are multiples of the vector width); the lane that
+// owns the lower vector rotates and writes both.  Four vectors per lane in flight.
+template <bool BF16>
+__device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict__ dst, const GatherArgs& g,
+                                 const float2* __restrict__ cs, int lane) {
+  using IO = Vec16<BF16>;
+  constexpr int N = IO::N;
+  const uint4* s = reinterpret_cast<const uint4*>(src);
+  uint4* d = reinterpret_cast<uint4*>(dst);
+  const int n = g.row_bytes >> 4;
+  const int vph = g.d / N;  // vectors per head
+  const int c0 = g.rope_c0, np = g.rope_pairs, np2 = 2 * g.rope_pairs;
+  const int half = np / N;
+  for (int base = lane; base < n; base += 128) {
+    uint4 v[4], w[4];
+    int kind[4], ch[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int c = base + 32 * u;
+      kind[u] = -1;  // past the row
+      ch[u] = 0;
+      if (c < n) {
+        ch[u] = (c % vph) * N;
+        if (g.rope_interleaved)
+          kind[u] = (ch[u] + N > c0 && ch[u] < c0 + np2) ? 1 : 0;
+        else
+          kind[u] = (ch[u] >= c0 && ch[u] < c0 + np) ? 2 : ((ch[u] >= c0 + np && ch[u] < c0 + np2) ? 3 : 0);
+        if (kind[u] != 3) v[u] = __ldg(s + c);
+        if (kind[u] == 2) w[u] = __ldg(s + c + half);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int c = base + 32 * u;
+      if (kind[u] == 0) {
+        d[c] = v[u];
+      } else if (kind[u] == 1) {
+        float x[N];
+        IO::unpack(v[u], x);
+#pragma unroll
+        for (int e = 0; e < N; e += 2) {
+          const int che = ch[u] + e;
+          if (che >= c0 && che < c0 + np2) rotate_pair(x[e], x[e + 1], cs[(che - c0) >> 1]);
+        }
+        d[c] = IO::pack(x);
+      } else if (kind[u] == 2) {
+        float x[N], y[N];
+        IO::unpack(v[u], x);
+        IO::unpack(w[u], y);
+#pragma unroll
+        for (int e = 0; e < N; ++e) rotate_pair(x[e], y[e], cs[ch[u] - c0 + e]);
+        d[c] = IO::pack(x);
+        d[c + half] = IO::pack(y);
+      }
+    }
+  }
+}
+
+// Copies every active slot's K and V rows (one warp per token row, rows ordered
+// (active slot, K|V, layer, token)) from its slab into the slot's cache segment.
+__device__ inline void gather_slots(const GatherArgs& g, int k, const GatherPlan& p) {
+  int act[CRC_MAX_K];
+  int n_act = 0;
+  for (int r = 0; r < k; ++r)
+    if (p.chunk[r] >= 0 && g.slot_offset[r] >= 0) act[n_act++] = r;
+  const int64_t rows_per_kv = (int64_t)g.L * g.Nc;
+  const int64_t total = (int64_t)n_act * 2 * rows_per_kv;
+  const int lane = threadIdx.x & 31;
+  const int gwarp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int nwarps = (gridDim.x * blockDim.x) >> 5;
+  for (int64_t row = gwarp; row < total; row += nwarps) {
+    const int ai = (int)(row / (2 * rows_per_kv));
+    int64_t rem = row - (int64_t)ai * 2 * rows_per_kv;
+    const int kv = (int)(rem / rows_per_kv);
+    rem -= kv * rows_per_kv;
+    const int l = (int)(rem / g.Nc);
+    const int t = (int)(rem - (int64_t)l * g.Nc);
+    const int r = act[ai];
+    const int64_t slab = p.chunk[r] % g.num_slabs;
+    const char* src = g.pool + slab * g.slab_bytes + kv * g.kv_bytes + rem * g.row_bytes;
+    char* dst = (kv ? g.cache_v : g.cache_k) + l * g.cache_layer_stride +
+                (int64_t)(g.slot_offset[r] + t) * g.cache_token_stride;
+    if (kv == 0 && p.rotate[r]) {
+      if (g.elem_bytes == 2)
+        copy_row_rotated<true>(src, dst, g, p.cs[r], lane);
+      else
+        copy_row_rotated<false>(src, dst, g, p.cs[r], lane);
+    } else {
+      warp_copy_row(src, dst, nullptr, g.row_bytes, lane);
+    }
+  }
+}
+
+}  // namespace crc

@@ -75,23 +75,13 @@ struct CacheUpdateArgs {
 };
 cudaError_t launch_cache_update(const CacheUpdateArgs& a, cudaStream_t s);
 
-struct RetrieveArgs {
-  FrameSet cur;
-  const double* centre;
-  const double* view;
-  int32_t count;
-  int32_t n;
-  double E, w_v, tau_c, cos_tau_v;
-  int32_t delta, k, ext_first, ext_min;
-  int32_t* d_idx;
-  double* d_score;
-  int32_t* d_count;
-  // gather (skipped when cache_k is null)
-  const char* pool;
+// Slab-to-cache gather of the retrieved slots, with the optional temporal RoPE
+// re-positioning of the keys (crc_rope).
+struct GatherArgs {
+  const char* pool;     // [num_slabs][2][L][Nc][H][d]; null disables the gather
   int32_t num_slabs;
   int64_t slab_bytes;
   int64_t kv_bytes;     // bytes of the K half of a slab
-  int64_t layer_bytes;  // bytes of one layer inside a slab half
   char* cache_k;
   char* cache_v;
   int64_t cache_layer_stride;  // bytes
@@ -99,9 +89,37 @@ struct RetrieveArgs {
   int32_t slot_offset[CRC_MAX_K];  // token offset of slot r's segment, -1 if none
   int32_t L;
   int32_t Nc;
-  int32_t row_bytes;
+  int32_t row_bytes;    // H*d*elem
+  int32_t d;            // head dim
+  int32_t elem_bytes;   // 2 (bf16) or 4 (fp32)
+  int32_t F;
+  // rope (rope_pairs = 0: plain copy)
+  int32_t rope_pairs, rope_c0, rope_interleaved;
+  int32_t rope_pos_slot0, rope_pos_stride, rope_frame_pos0;
+  double rope_omega[CRC_MAX_ROPE_PAIRS];  // theta^(-i/pairs)
+};
+
+struct RetrieveArgs {
+  FrameSet cur;
+  const double* centre;
+  const double* view;
+  int32_t count;
+  int32_t n;
+  double E, w_v, tau_c, cos_tau_v;
+  int32_t delta, k, ext_first, ext_min, exclude_sink;
+  int32_t* d_idx;
+  double* d_score;
+  int32_t* d_count;
+  GatherArgs g;
 };
 cudaError_t launch_retrieve(const RetrieveArgs& a, cudaStream_t s);
+
+struct GatherOnlyArgs {
+  const int32_t* d_idx;  // [k] chunk per slot (negative = empty)
+  int32_t k;
+  GatherArgs g;
+};
+cudaError_t launch_gather(const GatherOnlyArgs& a, cudaStream_t s);
 
 struct CorrespondArgs {
   FrameSet cur;

@@ -11,7 +11,7 @@
 #include <float.h>
 #include <limits.h>
 
-#include "copy.cuh"
+#include "gather.cuh"
 #include "internal.cuh"
 
 namespace crc {
@@ -47,7 +47,7 @@ __global__ void __launch_bounds__(256) retrieve_gather_kernel(const __grid_const
   __shared__ double sh_cn[3], sh_vn[3];
   __shared__ double red_s[8];
   __shared__ int red_j[8];
-  __shared__ int slot_chunk[CRC_MAX_K];
+  __shared__ GatherPlan plan;
   __shared__ double slot_score[CRC_MAX_K];
   __shared__ int sh_count;
   const int tid = threadIdx.x;
@@ -77,7 +77,8 @@ __global__ void __launch_bounds__(256) retrieve_gather_kernel(const __grid_const
     for (int j = tid; j < a.count; j += blockDim.x) {
       double s, dist, dot;
       score_entry(a.centre, a.view, j, cn, vn, a.E, a.w_v, s, dist, dot);
-      const bool adm = (dist <= a.tau_c) && (dot >= a.cos_tau_v) && (a.n - j >= a.delta);
+      const bool adm = (dist <= a.tau_c) && (dot >= a.cos_tau_v) && (a.n - j >= a.delta) &&
+                       !(a.exclude_sink && j == 0);
       const bool after = first || cand_less(ps, pj, s, j);
       if (adm && after && cand_less(s, j, bs, bj)) {
         bs = s;
@@ -108,7 +109,7 @@ __global__ void __launch_bounds__(256) retrieve_gather_kernel(const __grid_const
     __syncthreads();
     if (bj == INT_MAX) break;  // block-uniform
     if (tid == 0) {
-      slot_chunk[r] = bj;
+      plan.chunk[r] = bj;
       slot_score[r] = bs;
     }
     ps = bs;
@@ -119,58 +120,56 @@ __global__ void __launch_bounds__(256) retrieve_gather_kernel(const __grid_const
   if (tid == 0) {
     for (int r = count; r < a.k; ++r) {
       const int e = a.ext_first - (r - count);
-      slot_chunk[r] = (a.ext_first >= 0 && e >= a.ext_min) ? e : -1;
+      plan.chunk[r] = (a.ext_first >= 0 && e >= a.ext_min) ? e : -1;
       slot_score[r] = __longlong_as_double(0x7ff0000000000000LL);  // +inf
     }
     sh_count = count;
     if (blockIdx.x == 0) {
       for (int r = 0; r < a.k; ++r) {
-        a.d_idx[r] = slot_chunk[r];
+        a.d_idx[r] = plan.chunk[r];
         if (a.d_score) a.d_score[r] = slot_score[r];
       }
       *a.d_count = count;
     }
   }
   __syncthreads();
-  if (a.cache_k == nullptr) return;
-
-  // gather: one warp per token row; rows ordered (active slot, kv, layer, token)
-  int act_slot[CRC_MAX_K];
-  int n_act = 0;
-  for (int r = 0; r < a.k; ++r)
-    if (slot_chunk[r] >= 0 && a.slot_offset[r] >= 0) act_slot[n_act++] = r;
-  const int64_t rows_per_kv = (int64_t)a.L * a.Nc;
-  const int64_t total = (int64_t)n_act * 2 * rows_per_kv;
-  const int gwarp = (blockIdx.x * blockDim.x + tid) >> 5;
-  const int nwarps = (gridDim.x * blockDim.x) >> 5;
-  for (int64_t row = gwarp; row < total; row += nwarps) {
-    const int ai = (int)(row / (2 * rows_per_kv));
-    int64_t rem = row - (int64_t)ai * 2 * rows_per_kv;
-    const int kv = (int)(rem / rows_per_kv);
-    rem -= kv * rows_per_kv;
-    const int l = (int)(rem / a.Nc);
-    const int t = (int)(rem - (int64_t)l * a.Nc);
-    const int r = act_slot[ai];
-    const int slab = slot_chunk[r] % a.num_slabs;
-    const char* src = a.pool + slab * a.slab_bytes + kv * a.kv_bytes + rem * a.row_bytes;
-    char* dst = (kv ? a.cache_v : a.cache_k) + l * a.cache_layer_stride +
-                (int64_t)(a.slot_offset[r] + t) * a.cache_token_stride;
-    warp_copy_row(src, dst, nullptr, a.row_bytes, lane);
-  }
+  if (a.g.pool == nullptr) return;
+  plan_rope(a.g, a.k, plan);
+  gather_slots(a.g, a.k, plan);
 }
 
+// The gather alone, for a cache that mirrors the retrieved slots of a step.
+__global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherOnlyArgs a) {
+  __shared__ GatherPlan plan;
+  if (threadIdx.x < a.k) plan.chunk[threadIdx.x] = a.d_idx[threadIdx.x];
+  __syncthreads();
+  plan_rope(a.g, a.k, plan);
+  gather_slots(a.g, a.k, plan);
+}
+
+namespace {
+
+// One warp per row; at most four CTAs of 256 threads per SM, grid-stride beyond that.
+int gather_blocks(int k, const GatherArgs& g) {
+  const int64_t rows = 2LL * k * g.L * g.Nc;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (rows + 7) / 8;
+  int blocks = (int)(want < (int64_t)sms * 4 ? want : (int64_t)sms * 4);
+  return blocks < 1 ? 1 : blocks;
+}
+
+}  // namespace
+
 cudaError_t launch_retrieve(const RetrieveArgs& a, cudaStream_t s) {
-  int blocks = 1;
-  if (a.cache_k) {
-    const int64_t rows = 2LL * a.k * a.L * a.Nc;
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int64_t want = (rows + 7) / 8;
-    blocks = (int)(want < (int64_t)sms * 4 ? want : (int64_t)sms * 4);
-    if (blocks < 1) blocks = 1;
-  }
+  const int blocks = a.g.pool ? gather_blocks(a.k, a.g) : 1;
   retrieve_gather_kernel<<<blocks, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const GatherOnlyArgs& a, cudaStream_t s) {
+  gather_kernel<<<gather_blocks(a.k, a.g), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -10,8 +10,14 @@ without any host synchronisation:
   crc_retrieve        Eq. 1 over chunks 0..n, gates (distance, angle, gap delta),
                       top-k gather into the retrieved slots; an empty admissible set
                       extends the window with the next-older chunks n-W, n-W-1, ...
+  crc_gather          (optional) the same slots into the control-branch cache
   crc_correspond      Eq. 3-4 for every query of chunk n in every retrieved frame
   crc_biased_attention  Eq. 2 over all layers of the call
+
+With `rope_pairs` > 0 the retrieved chunks' keys (cached with their rotary
+embedding at the frame positions where they were produced, frame f of chunk j at
+j F + f) are re-packed at the positions just before the recent window: slot r
+at (n - W + 1 - k + r) F + f at step n (Sec. 4.2 "Cache packing").
 
 Everything numeric happens in the CUDA kernels; this module only decides which
 cache region each chunk occupies and which segments are live at step n.
@@ -49,6 +55,13 @@ class StreamConfig:
     sigma: float
     eps: float
     dtype: torch.dtype = torch.bfloat16
+    # temporal RoPE re-positioning of retrieved keys (0 pairs: off)
+    rope_pairs: int = 0
+    rope_channel0: int = 0
+    rope_theta: float = 10000.0
+    rope_interleaved: bool = True
+    # control-branch mirror cache with its own layer count (0: none)
+    control_L: int = 0
 
     @property
     def Nc(self) -> int:
@@ -77,6 +90,13 @@ class ChunkStream:
         self.valid = torch.zeros(c.Nc, S, dtype=torch.uint8, device=device)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
         self.params = api.retrieval_params(c.E, c.w_v, c.tau_c, c.cos_tau_v, c.delta, c.k)
+        self.control_shape = None
+        if c.control_L > 0:
+            # the control branch keeps its own slab pool and cache; poses and depth live in the main bank
+            self.control_shape = api.shape(c.control_L, c.H, c.d, c.F, c.h, c.w, c.dtype)
+            self.control_bank = api.Bank(c.capacity, c.F, c.h, c.w, c.control_L, c.H, c.d, c.dtype, c.num_slabs,
+                                         device=device)
+            self.control_cache = api.Cache.empty(c.control_L, c.n_keys, c.H, c.d, c.dtype, [], device=device)
 
     # ---- layout -----------------------------------------------------------
     def slot_offset(self, r: int) -> int:
@@ -97,6 +117,15 @@ class ChunkStream:
             segs.append((self.window_offset(q), c.Nc if present else 0, api.SEG_WINDOW, q))
         return segs
 
+    def rope(self, n: int):
+        """Re-positioning of step n: slot r just before the window's oldest chunk."""
+        c = self.cfg
+        if c.rope_pairs <= 0:
+            return None
+        first_window_chunk = max(1, n - c.window + 1)
+        return api.rope_params(c.rope_channel0, c.rope_pairs, c.rope_theta, c.rope_interleaved,
+                               pos_slot0=(first_window_chunk - c.k) * c.F, pos_stride=c.F, frame_pos0=0)
+
     def ext_first(self, n: int) -> int:
         """Newest chunk that is neither in the window nor the sink (-1 if none)."""
         e = n - self.cfg.window
@@ -104,14 +133,23 @@ class ChunkStream:
 
     # ---- one chunk step ---------------------------------------------------
     def step(self, n: int, frames: np.ndarray, depth: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
-             q: torch.Tensor, o: torch.Tensor, lse: Optional[torch.Tensor] = None, stream=None) -> None:
+             q: torch.Tensor, o: torch.Tensor, lse: Optional[torch.Tensor] = None, stream=None,
+             k_ctl: Optional[torch.Tensor] = None, v_ctl: Optional[torch.Tensor] = None) -> None:
         c = self.cfg
         woff = 0 if n == 0 else self.window_offset(n % c.window)
         self.cache.segments = self.segments(n)
         api.crc_cache_update(self.bank, self.shape, n, frames, depth, k_new, v_new, self.cache, woff, stream)
+        if self.control_shape is not None:
+            self.control_cache.segments = self.cache.segments
+            api.crc_cache_update(self.control_bank, self.control_shape, n, frames, depth, k_ctl, v_ctl,
+                                 self.control_cache, woff, stream)
         params = api.retrieval_params(c.E, c.w_v, c.tau_c, c.cos_tau_v, c.delta, c.k, self.ext_first(n), 1)
+        rope = self.rope(n)
         api.crc_retrieve(self.bank, n + 1, self.shape, frames, n, params, self.cache, self.idx, self.score,
-                         self.count, stream)
+                         self.count, stream, rope=rope)
+        if self.control_shape is not None:
+            api.crc_gather(self.control_shape, self.control_bank.kv, self.idx, c.k, self.control_cache, rope=rope,
+                           stream=stream)
         api.crc_correspond(self.shape, frames, depth, self.bank, self.idx, self.count, c.k, c.eps, self.uv,
                            self.cell, self.valid, stream)
         api.crc_biased_attention(self.shape, q, self.cache, o, lse, self.uv, self.valid, c.k, self.idx, c.lam,

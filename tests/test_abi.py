@@ -58,9 +58,10 @@ _LAYOUT_C = r"""
 #define P(T) printf(#T " %zu\n", sizeof(T));
 #define O(T, f) printf(#T "." #f " %zu\n", offsetof(T, f));
 int main(void) {
-  P(crc_frame) P(crc_shape) P(crc_tensor) P(crc_segment) P(crc_cache) P(crc_bank) P(crc_retrieval)
+  P(crc_frame) P(crc_shape) P(crc_tensor) P(crc_segment) P(crc_cache) P(crc_bank) P(crc_retrieval) P(crc_rope)
   O(crc_cache, v) O(crc_cache, n_keys) O(crc_cache, seg) O(crc_bank, frames) O(crc_bank, kv)
-  O(crc_retrieval, delta) O(crc_retrieval, ext_min) O(crc_shape, dtype) O(crc_tensor, stride_head)
+  O(crc_retrieval, delta) O(crc_retrieval, ext_min) O(crc_retrieval, exclude_sink) O(crc_shape, dtype)
+  O(crc_tensor, stride_head) O(crc_rope, frame_pos0) O(crc_rope, theta)
   return 0;
 }
 """
@@ -83,7 +84,9 @@ def test_ctypes_layout_matches_header():
         "crc_frame": C.sizeof(_abi.crc_frame), "crc_shape": C.sizeof(_abi.crc_shape),
         "crc_tensor": C.sizeof(_abi.crc_tensor), "crc_segment": C.sizeof(_abi.crc_segment),
         "crc_cache": C.sizeof(_abi.crc_cache), "crc_bank": C.sizeof(_abi.crc_bank),
-        "crc_retrieval": C.sizeof(_abi.crc_retrieval),
+        "crc_retrieval": C.sizeof(_abi.crc_retrieval), "crc_rope": C.sizeof(_abi.crc_rope),
+        "crc_retrieval.exclude_sink": _abi.crc_retrieval.exclude_sink.offset,
+        "crc_rope.frame_pos0": _abi.crc_rope.frame_pos0.offset, "crc_rope.theta": _abi.crc_rope.theta.offset,
         "crc_cache.v": _abi.crc_cache.v.offset, "crc_cache.n_keys": _abi.crc_cache.n_keys.offset,
         "crc_cache.seg": _abi.crc_cache.seg.offset, "crc_bank.frames": _abi.crc_bank.frames.offset,
         "crc_bank.kv": _abi.crc_bank.kv.offset, "crc_retrieval.delta": _abi.crc_retrieval.delta.offset,

@@ -108,3 +108,67 @@ def test_loop_stream_200_steps():
             lg = lse[layers][:, heads].cpu().numpy()[:, :, rows]
             assert np.abs(lg - lo).max() <= 1e-3
     assert n_closed >= 40  # the loop closes after one lap and stays closed
+
+
+def test_loop_stream_with_rope_repositioning_and_control_mirror():
+    # the same 200-step loop with re-positioned retrieved keys and a control-branch cache
+    # mirroring the retrieved slots (small head count; retrieval and gathers are what is checked)
+    wl = synth.make_workload(5)
+    cfg = crs.StreamConfig(L=2, H=2, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2, capacity=wl.bank_size,
+                           num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c, cos_tau_v=wl.cos_tau_v,
+                           delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps, rope_pairs=22,
+                           rope_interleaved=True, control_L=1)
+    st = crs.ChunkStream(cfg)
+    Nc = cfg.Nc
+    g = torch.Generator(device="cuda").manual_seed(6)
+    s = wl.qkv_scale
+    nbuf = 3
+
+    def rnd(L):
+        return (torch.randn(L, Nc, cfg.H, cfg.d, generator=g, device="cuda") * s).bfloat16()
+
+    kv = [(rnd(cfg.L), rnd(cfg.L)) for _ in range(nbuf)]
+    ctl = [(rnd(1), rnd(1)) for _ in range(nbuf)]
+    q = rnd(cfg.L)
+    o = torch.empty_like(q)
+
+    def slab_owner(slab, n):
+        return slab + ((n - slab) // cfg.num_slabs) * cfg.num_slabs
+
+    def rope_of(n):
+        r = st.rope(n)
+        return dict(channel0=r.channel0, pairs=r.pairs, theta=r.theta, interleaved=True, pos_slot0=r.pos_slot0,
+                    pos_stride=r.pos_stride, frame_pos0=r.frame_pos0, F=cfg.F)
+
+    checked = 0
+    for n in range(wl.bank_size):
+        fr = wl.bank_frames[n]
+        dep = torch.from_numpy(wl.depth_of(n)).cuda()
+        st.step(n, synth.frame_records(fr), dep, kv[n % nbuf][0], kv[n % nbuf][1], q, o,
+                k_ctl=ctl[n % nbuf][0], v_ctl=ctl[n % nbuf][1])
+        torch.cuda.synchronize()
+        assert st.status.item() == 0
+        _, _, oc, slots = _gpu.oracle_retrieve(wl, bank_count=n + 1, n=n, ext_first=st.ext_first(n), ext_min=1)
+        np.testing.assert_array_equal(st.idx.cpu().numpy(), slots)
+        # the window is never rotated: newest chunks byte-exact in both caches
+        for m in range(max(1, n - 1), n + 1):
+            off = st.window_offset(m % 2)
+            assert torch.equal(st.cache.k[:, off:off + Nc], kv[m % nbuf][0])
+            assert torch.equal(st.control_cache.k[:, off:off + Nc], ctl[m % nbuf][0])
+        if not (n % 10 == 0 or 150 <= n <= 155):
+            continue
+        for r, j in enumerate(slots):
+            if j < 0:
+                continue
+            owner = slab_owner(j % cfg.num_slabs, n) % nbuf
+            off = st.slot_offset(r)
+            for cache, src in ((st.cache, kv[owner]), (st.control_cache, ctl[owner])):
+                host = np.stack([src[0].double().cpu().numpy(), src[1].double().cpu().numpy()])
+                # slot r holds chunk j, read from a one-slab pool holding its K/V buffers
+                ref = oracle.gather(host[None], np.array([-1] * r + [j]), 1, rope=rope_of(n))[r]
+                got = cache.k[:, off:off + Nc]
+                np.testing.assert_allclose(got.double().cpu().numpy(), ref[0], rtol=2.0 ** -8,
+                                           atol=1e-6 * float(np.abs(host).max()))
+                assert torch.equal(cache.v[:, off:off + Nc], src[1])
+                checked += 1
+    assert checked >= 40
