@@ -272,9 +272,12 @@ def key_table(segments: Sequence[Tuple[int, int, int, int]], n_keys: int, h: int
 
 
 def bias_matrix(uv: np.ndarray, valid: np.ndarray, rows: np.ndarray, src: np.ndarray, ux: np.ndarray,
-                uy: np.ndarray, sigma: float) -> np.ndarray:
+                uy: np.ndarray, sigma: float, form: str = "eq2") -> np.ndarray:
     """Eq. 2 bias B_s(p, k) = -||u_k - u^_s(p)||^2 / (2 sigma^2) for query rows `rows`;
-    zero on columns without a source frame and for invalid correspondences."""
+    zero on columns without a source frame and for invalid correspondences.
+
+    form = "gaussian" is the opt-in additive variant exp(-||u_k - u^_s(p)||^2 / (2 sigma^2))
+    (a bonus that peaks at the correspondence) in place of Eq. 2's quadratic penalty."""
     B = np.zeros((rows.shape[0], src.shape[0]))
     for s in np.unique(src[src >= 0]):
         cols = np.nonzero(src == s)[0]
@@ -282,6 +285,10 @@ def bias_matrix(uv: np.ndarray, valid: np.ndarray, rows: np.ndarray, src: np.nda
         uhy = uv[rows, s, 1].astype(np.float64)[:, None]
         d2 = (ux[cols][None, :] - uhx) ** 2 + (uy[cols][None, :] - uhy) ** 2
         b = -d2 / (2.0 * sigma * sigma)
+        if form == "gaussian":
+            b = np.exp(b)
+        elif form != "eq2":
+            raise ValueError(form)
         b = np.where(valid[rows, s].astype(bool)[:, None], b, 0.0)
         B[:, cols] = b
     return B
@@ -291,8 +298,9 @@ def attention(Q: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, uv: np.ndarray, val
               segments, h: int, w: int, F: int, lam: float, sigma: float,
               slot_chunks: Optional[np.ndarray] = None, rows: Optional[np.ndarray] = None,
               layers: Optional[Sequence[int]] = None, heads: Optional[Sequence[int]] = None,
-              row_block: int = 1024):
+              row_block: int = 1024, bias_form: str = "eq2"):
     """Eq. 2: O_p = sum_k softmax_k(A_pk) V_k with A_pk = q_p.k_k / sqrt(d) + lam B_s(p, k).
+    bias_form selects the bias of `bias_matrix` (Eq. 2, or the opt-in additive Gaussian).
 
     Q [L, Nq, H, d], Kc/Vc [L, Nk, H, d] (values as given, widened to fp64),
     uv [Nq, S, 2], valid [Nq, S].  Softmax runs over the active keys only, in two
@@ -311,7 +319,7 @@ def attention(Q: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, uv: np.ndarray, val
     scale = 1.0 / math.sqrt(d)
     for b0 in range(0, rows.shape[0], row_block):
         rb = rows[b0:b0 + row_block]
-        lamB = lam * bias_matrix(uv, valid, rb, src[act], ux[act], uy[act], sigma)
+        lamB = lam * bias_matrix(uv, valid, rb, src[act], ux[act], uy[act], sigma, bias_form)
         for li, l in enumerate(layers):
             for hi, hh in enumerate(heads):
                 q = Q[l, rb, hh, :].astype(np.float64)

@@ -447,6 +447,43 @@ def test_bias_vanishes_at_correspondence_and_concentrates_as_lambda_grows():
     np.testing.assert_array_equal(Wb[0, 1:], W0[0, 1:])
 
 
+def test_additive_gaussian_form_raises_weights_near_the_correspondence():
+    # opt-in variant: A = q.k/sqrt(d) + beta exp(-d^2 / (2 sigma^2)) on retrieved keys with a valid pair
+    h, w, F = 3, 4, 2
+    Nc = F * h * w
+    segs = [(0, Nc, 0, 0), (Nc, Nc, 1, 0)]
+    Nk = 2 * Nc
+    Vid = np.eye(Nk)[None, :, None, :]
+    Kp = np.zeros((1, Nk, 1, Nk))
+    Qp = np.zeros((1, Nc, 1, Nk))  # all logits equal without bias
+    uv = np.zeros((Nc, F, 2))
+    valid = np.zeros((Nc, F), bool)
+    uv[0, 1] = (2.0, 1.0)
+    valid[0, 1] = True
+    target = Nc + 1 * h * w + 1 * w + 2
+    beta, sigma = 1.3, 0.9
+    Wg, _ = oracle.attention(Qp, Kp, Vid, uv, valid, segs, h, w, F, lam=beta, sigma=sigma, bias_form="gaussian")
+    # at the correspondence the weight is e^beta times a sink key's
+    assert Wg[0, 0, 0, target] / Wg[0, 0, 0, 0] == pytest.approx(math.exp(beta), rel=1e-14)
+    # one cell away: e^(beta exp(-1 / (2 sigma^2)))
+    assert Wg[0, 0, 0, target - 1] / Wg[0, 0, 0, 0] == pytest.approx(
+        math.exp(beta * math.exp(-1.0 / (2 * sigma * sigma))), rel=1e-14)
+    # the other source frame (no valid pair for query 0) and the other queries are untouched
+    assert Wg[0, 0, 0, Nc] == pytest.approx(Wg[0, 0, 0, 0], rel=1e-14)
+    W0, _ = oracle.attention(Qp, Kp, Vid, uv, valid, segs, h, w, F, lam=0.0, sigma=sigma, bias_form="gaussian")
+    np.testing.assert_array_equal(Wg[0, 1:], W0[0, 1:])
+    # far from the correspondence the bonus vanishes: a 1 x 40 frame, keys 30 cells away
+    h2, w2, F2 = 1, 40, 1
+    segs2 = [(0, 40, 0, 0), (40, 40, 1, 0)]
+    uv2 = np.zeros((40, 1, 2))
+    valid2 = np.ones((40, 1), bool)
+    W2, _ = oracle.attention(np.zeros((1, 40, 1, 80)), np.zeros((1, 80, 1, 80)), np.eye(80)[None, :, None, :],
+                             uv2, valid2, segs2, h2, w2, F2, lam=beta, sigma=1.0, bias_form="gaussian")
+    assert W2[0, 0, 0, 40 + 30] / W2[0, 0, 0, 0] == pytest.approx(1.0, abs=1e-12)
+    with pytest.raises(ValueError):
+        oracle.attention(Qp, Kp, Vid, uv, valid, segs, h, w, F, lam=beta, sigma=sigma, bias_form="other")
+
+
 def test_empty_retrieved_slot_is_masked():
     Q, Kc, Vc, uv, valid, segs, h, w, F = _tiny_attn_inputs(seed=5)
     Nc = F * h * w
