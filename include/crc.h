@@ -279,7 +279,17 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
 
 /* crc_biased_attention flags */
 #define CRC_ATTN_DEFAULT 0
-#define CRC_ATTN_SIMT 1  /* force the SIMT kernel (fp32 arithmetic) for any dtype */
+#define CRC_ATTN_SIMT 1      /* force the SIMT kernel (fp32 arithmetic) for any dtype */
+#define CRC_ATTN_GAUSSIAN 2  /* opt-in: additive Gaussian bias lambda exp(-||u_k - u^||^2 / (2 sigma^2))
+                                on the biased columns instead of Eq. 2's quadratic penalty
+                                (a bonus that peaks at the correspondence; runs on the SIMT kernel) */
+#define CRC_ATTN_SKIP_FAR 4  /* opt-in approximation (tensor-core kernel, Eq. 2 form): a KV tile of a
+                                retrieved frame is skipped for a block of 256 queries when every one of
+                                them has a valid correspondence in that frame and the distance from the
+                                box of those correspondences to the tile's key cells is at least
+                                sigma sqrt(128 ln 2 / lambda), i.e. the bias scales each skipped weight by
+                                at most 2^-64.  Only retrieved tiles are skipped, and only when the cache
+                                has other active keys. */
 
 /*
  * crc_biased_attention — Sec. 4.3, Eq. 2, for every layer l < L, head and query p:
@@ -300,9 +310,9 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
  *   d_status  device int32 or NULL: set non-zero if a kernel gave up waiting on
  *             an internal pipeline barrier (the output is then not valid).
  * bf16 (d = 128) runs on the tcgen05 tensor-core kernel with fp32 softmax and
- * accumulation; fp32 (or CRC_ATTN_SIMT) runs the SIMT kernel in fp32.
- * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE, CRC_ERR_UNSUPPORTED (dtype, d,
- * alignment, device without sm_103a), CRC_ERR_CUDA.
+ * accumulation; fp32, CRC_ATTN_SIMT or CRC_ATTN_GAUSSIAN run the SIMT kernel in fp32.
+ * Errors: CRC_ERR_INVALID_ARG (also unknown flag bits), CRC_ERR_SHAPE,
+ * CRC_ERR_UNSUPPORTED (dtype, d, alignment, device without sm_103a), CRC_ERR_CUDA.
  */
 crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_cache* cache, crc_tensor o,
                                 float* d_lse, int32_t n_q, const float* d_uv, const uint8_t* d_valid, int32_t k,

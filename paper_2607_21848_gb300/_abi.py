@@ -32,6 +32,8 @@ CRC_MAX_ROPE_PAIRS = 64
 
 CRC_ATTN_DEFAULT = 0
 CRC_ATTN_SIMT = 1
+CRC_ATTN_GAUSSIAN = 2
+CRC_ATTN_SKIP_FAR = 4
 
 
 class crc_frame(C.Structure):

@@ -23,6 +23,8 @@ SEG_RETRIEVED = _abi.CRC_SEG_RETRIEVED
 SEG_WINDOW = _abi.CRC_SEG_WINDOW
 ATTN_DEFAULT = _abi.CRC_ATTN_DEFAULT
 ATTN_SIMT = _abi.CRC_ATTN_SIMT
+ATTN_GAUSSIAN = _abi.CRC_ATTN_GAUSSIAN
+ATTN_SKIP_FAR = _abi.CRC_ATTN_SKIP_FAR
 
 
 def _dtype_code(dt: torch.dtype) -> int:

@@ -326,12 +326,16 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
   if (n_q != nc) return CRC_ERR_SHAPE;
   if (k < 0 || k > CRC_MAX_K || !isfinite(lambda) || lambda < 0.f || !(sigma > 0.f) || !isfinite(sigma))
     return CRC_ERR_INVALID_ARG;
-  bool any_ret = false;
-  for (int g = 0; g < cache->nseg; ++g)
+  if (flags & ~(CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN | CRC_ATTN_SKIP_FAR)) return CRC_ERR_INVALID_ARG;
+  bool any_ret = false, any_other = false;
+  for (int g = 0; g < cache->nseg; ++g) {
     if (cache->seg[g].kind == CRC_SEG_RETRIEVED && cache->seg[g].length > 0) {
       any_ret = true;
       if (cache->seg[g].slot >= k) return CRC_ERR_SHAPE;
+    } else if (cache->seg[g].length > 0) {
+      any_other = true;
     }
+  }
   if (any_ret && (!d_uv || !d_valid)) return CRC_ERR_INVALID_ARG;
   if (q.stride_head < shape->d || q.stride_token < (int64_t)shape->H * q.stride_head ||
       o.stride_head < shape->d || o.stride_token < (int64_t)shape->H * o.stride_head)
@@ -370,8 +374,13 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
   a.sigma = sigma;
   a.dtype = shape->dtype;
   a.status = d_status;
+  a.bias_form = (flags & CRC_ATTN_GAUSSIAN) ? 1 : 0;
+  // skipped weights are scaled by at most 2^-64: lambda d^2 / (2 sigma^2) >= 64 ln 2
+  a.skip_far = (flags & CRC_ATTN_SKIP_FAR) && lambda > 0.f && any_ret && any_other && d_valid ? 1 : 0;
+  a.skip_d2 = lambda > 0.f ? (float)(2.0 * (double)sigma * (double)sigma * 64.0 * 0.6931471805599453 / (double)lambda)
+                           : INFINITY;
   cudaError_t e;
-  if (shape->dtype == CRC_BF16 && !(flags & CRC_ATTN_SIMT)) {
+  if (shape->dtype == CRC_BF16 && !(flags & (CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN))) {
     e = crc::launch_attn_tc(a, s);
     if (e == cudaErrorNotSupported) return CRC_ERR_UNSUPPORTED;
   } else {

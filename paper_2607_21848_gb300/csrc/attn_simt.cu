@@ -5,7 +5,8 @@
 // One CTA (4 warps) owns 16 query rows of one (layer, head) and streams the
 // key/value tiles of 32 keys through shared memory; lane l scores key l of the
 // tile for each of its warp's 4 queries, adds lambda*B from the correspondence of
-// that query in the key's source frame, and the warp keeps an online softmax.
+// that query in the key's source frame (Eq. 2, or the opt-in additive Gaussian
+// lambda exp(-d^2 / (2 sigma^2))), and the warp keeps an online softmax.
 // The bias is formed per (query, key) in registers and never stored.
 #include <cuda_bf16.h>
 #include <math.h>
@@ -56,6 +57,7 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const __grid_constant__ 
   }
   const float scale = rsqrtf((float)d);
   const float nb = a.lambda / (2.f * a.sigma * a.sigma);
+  const float ng = 1.f / (2.f * a.sigma * a.sigma);
   const int dpl = d / 32;  // output dims per lane
   float m[4], l[4], acc[4][kMaxD / 32];
 #pragma unroll
@@ -88,7 +90,10 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const __grid_constant__ 
         if (a.valid[pi]) {
           const float2 u = reinterpret_cast<const float2*>(a.uv)[pi];
           const float dx = ki.x - u.x, dy = ki.y - u.y;
-          logit -= nb * (dx * dx + dy * dy);
+          if (a.bias_form == 1)
+            logit += a.lambda * expf(-ng * (dx * dx + dy * dy));  // opt-in additive Gaussian
+          else
+            logit -= nb * (dx * dx + dy * dy);  // Eq. 2
         }
       }
       if (!ki.active) logit = -INFINITY;

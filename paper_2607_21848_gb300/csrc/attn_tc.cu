@@ -46,6 +46,7 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
+#include <limits.h>
 #include <math.h>
 #include <string.h>
 
@@ -92,7 +93,8 @@ constexpr int OFF_TILES = OFF_RB + NBB * AUG;
 constexpr int OFF_BAR = OFF_TILES + kMaxTiles * 12;
 constexpr int NBAR = 1 + 4 * ST + 3 * NQT + 1 + NQT + 2 * NBB;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
-constexpr int SMEM_BYTES = OFF_MISC + 64 + 1024;  // + slack for 1024-byte alignment
+constexpr int OFF_BOX = OFF_MISC + 64;  // per source frame: correspondence box of the CTA's queries
+constexpr int SMEM_BYTES = OFF_BOX + CRC_MAX_K * CRC_MAX_FRAMES * 5 * 4 + 1024;  // + slack for 1024-byte alignment
 static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 
 constexpr uint32_t TM_S = 0;    // S/P of tile x at column 128 x
@@ -222,6 +224,13 @@ __device__ __forceinline__ void aug_query_row(const Corr& c, float xc, float yc,
   w[7] = a3[2] | (bf16_bits(1.f) << 16);  // mask column
 }
 
+// fp32 <-> int keys with the same order, for shared-memory atomic min / max
+__device__ __forceinline__ int ord_key(float f) {
+  const int b = __float_as_int(f);
+  return b >= 0 ? b : b ^ 0x7fffffff;
+}
+__device__ __forceinline__ float ord_val(int k) { return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff); }
+
 __device__ __forceinline__ void fail(const TcParams& P, volatile int* abort_flag, int code) {
   *abort_flag = 1;
   if (P.a.status) atomicExch(P.a.status, code);
@@ -268,6 +277,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
+  // CRC_ATTN_SKIP_FAR: per source frame, whether every query of this CTA has a valid
+  // correspondence there, and the bounding box of those correspondences
+  int* box = reinterpret_cast<int*>(smem + OFF_BOX);  // [S][5]: x min, x max, y min, y max, all valid
+  const bool skip_far = a.skip_far != 0;
+  if (skip_far) {
+    for (int i = tid; i < a.S; i += kThreads) {
+      box[5 * i + 0] = INT_MAX;
+      box[5 * i + 1] = INT_MIN;
+      box[5 * i + 2] = INT_MAX;
+      box[5 * i + 3] = INT_MIN;
+      box[5 * i + 4] = 1;
+    }
+    __syncthreads();
+    const int rows = min(NQT * BM, a.Nq - q0);
+    for (int e = tid; e < rows * a.S; e += kThreads) {
+      const int rr = e / a.S, sf = e - rr * a.S;
+      const int64_t pi = (int64_t)(q0 + rr) * a.S + sf;
+      if (!a.valid[pi]) {
+        atomicAnd(&box[5 * sf + 4], 0);
+        continue;
+      }
+      const float2 u = reinterpret_cast<const float2*>(a.uv)[pi];
+      atomicMin(&box[5 * sf + 0], ord_key(u.x));
+      atomicMax(&box[5 * sf + 1], ord_key(u.x));
+      atomicMin(&box[5 * sf + 2], ord_key(u.y));
+      atomicMax(&box[5 * sf + 3], ord_key(u.y));
+    }
+    __syncthreads();
+  }
   if (warp == 0) {
     // KV tiles: each segment is cut into tiles of 128 keys from its start; retrieved
     // segments are cut per source frame, so that a tile has at most one frame
@@ -294,11 +332,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           ti.cls = (nact == BN && !ret) ? CLS_PLAIN : CLS_AUG;
           ti.pad = 0;
           ti.loc0 = (uint16_t)(t * BN);
+          bool keep = act;
+          if (skip_far && ret && act) {
+            // the tile's key cells against the box of this frame's correspondences
+            const int sf = sg.slot * a.F + rr;
+            if (box[5 * sf + 4] && box[5 * sf + 0] != INT_MAX) {
+              const int l0 = t * BN, l1 = l0 + nact - 1;
+              const int y0 = l0 / a.w, y1 = l1 / a.w;
+              const float kx0 = y0 == y1 ? (float)(l0 - y0 * a.w) : 0.f;
+              const float kx1 = y0 == y1 ? (float)(l1 - y1 * a.w) : (float)(a.w - 1);
+              const float dx = fmaxf(0.f, fmaxf(ord_val(box[5 * sf + 0]) - kx1, kx0 - ord_val(box[5 * sf + 1])));
+              const float dy = fmaxf(0.f, fmaxf(ord_val(box[5 * sf + 2]) - (float)y1, (float)y0 - ord_val(box[5 * sf + 3])));
+              keep = !(dx * dx + dy * dy >= a.skip_d2);
+            }
+          }
           const unsigned lt = (1u << lane) - 1u;
-          const unsigned m = __ballot_sync(0xffffffffu, act);
-          const unsigned ma = __ballot_sync(0xffffffffu, act && ti.cls == CLS_AUG);
+          const unsigned m = __ballot_sync(0xffffffffu, keep);
+          const unsigned ma = __ballot_sync(0xffffffffu, keep && ti.cls == CLS_AUG);
           ti.q = (uint16_t)(qa + __popc(ma & lt));
-          if (act) tiles[count + __popc(m & lt)] = ti;
+          if (keep) tiles[count + __popc(m & lt)] = ti;
           count += __popc(m);
           qa += __popc(ma);
         }

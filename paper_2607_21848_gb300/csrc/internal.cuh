@@ -157,6 +157,9 @@ struct AttnArgs {
   float sigma;
   int32_t dtype;
   int32_t* status;
+  int32_t bias_form;  // 0: Eq. 2 quadratic; 1: additive Gaussian (CRC_ATTN_GAUSSIAN)
+  int32_t skip_far;   // CRC_ATTN_SKIP_FAR in force (tensor-core kernel)
+  float skip_d2;      // squared grid distance beyond which a retrieved tile is skipped
 };
 cudaError_t launch_attn_simt(const AttnArgs& a, cudaStream_t s);
 // Returns cudaErrorNotSupported when the tensor-core kernel cannot take these arguments.

@@ -77,6 +77,18 @@ def _check_bf16(Og, lg, Oo, lo, rows=None):
         assert np.abs(lg - lo).max() <= 1e-3
 
 
+def _check_bf16_peaky(Og, Oo, Oabs):
+    """For outputs dominated by a few keys, where bf16 rounding alone exceeds 2e-2 x RMS:
+    max abs error <= 2e-2, and per element the rounding bound of the bf16 path -- P rounded
+    to bf16 (2^-9 relative per weight) and O rounded to bf16 (2^-9 relative), with a factor
+    2 margin: |O_gpu - O| <= 2^-8 (sum_k w_k |v_k| + |O|).  Oabs = the oracle run on |V|."""
+    err = np.abs(Og - Oo)
+    assert err.max() <= 2e-2, err.max()
+    bound = 2.0 ** -8 * (Oabs + np.abs(Oo)) + 1e-6
+    worst = (err / bound).max()
+    assert worst <= 1.0, worst
+
+
 def test_fp32_config1_matches_oracle_1e4():
     wl = synth.make_workload(1)
     idx, _, count, slots = _gpu.oracle_retrieve(wl)
@@ -196,3 +208,87 @@ def test_bf16_config4_full_size_sampled():
     rows = np.random.default_rng(2).choice(10800, 256, replace=False)
     rows.sort()
     _full_size(4, rows, [0], [0, 13, 39])
+
+
+# ---------------------------------------------------------------------------- opt-in modes
+def test_gaussian_form_fp32_and_bf16_match_oracle():
+    wl = synth.make_workload(1)
+    idx, _, count, slots = _gpu.oracle_retrieve(wl)
+    uv, cell, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
+    Q, Kc, Vc = synth.make_qkv(wl)
+    shp = api.shape(wl.L, wl.H, wl.d, wl.F, wl.h, wl.w, torch.float32)
+    beta = 1.5
+    Og, lg = _run_attn(shp, Q, Kc, Vc, wl.segments, uv.astype(np.float32), valid, wl.k, beta, wl.sigma,
+                       slot_chunk=slots, dtype=torch.float32, flags=api.ATTN_GAUSSIAN)
+    Oo, lo = oracle.attention(Q, Kc, Vc, uv.astype(np.float32).astype(np.float64), valid, wl.segments, wl.h, wl.w,
+                              wl.F, beta, wl.sigma, slot_chunks=slots, bias_form="gaussian")
+    assert np.abs(Og - Oo).max() <= 1e-4 and np.abs(lg - lo).max() <= 1e-4
+    Oq, _ = oracle.attention(Q, Kc, Vc, uv, valid, wl.segments, wl.h, wl.w, wl.F, beta, wl.sigma, slot_chunks=slots)
+    assert np.abs(Oq - Oo).max() > 1e-3  # the two bias forms differ here
+    # bf16 inputs take the SIMT kernel in this mode
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=21, L=1)
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=api.ATTN_GAUSSIAN)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0, bias_form="gaussian")
+    Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, 2.0, 1.0, bias_form="gaussian")
+    _check_bf16_peaky(Og, Oo, Oabs)
+    assert np.abs(lg - lo).max() <= 1e-3
+
+
+def test_unknown_attention_flags_are_rejected():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=22, L=1, H=1)
+    with pytest.raises(api.CrcError):
+        _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=8)
+
+
+def _skip_case(seed, far_logit=0.0, invalid_row=None):
+    # one frame of 32 x 8 tokens (two KV tiles per frame: rows 0-15 and 16-31), 256 queries in one
+    # CTA whose correspondences all lie in rows 0-9; the second tile is >= 7 rows away
+    g = np.random.default_rng(seed)
+    F, h, w, k = 1, 32, 8, 1
+    Nc = F * h * w
+    segs = [(0, Nc, api.SEG_SINK, 0), (Nc, Nc, api.SEG_RETRIEVED, 0), (2 * Nc, Nc, api.SEG_WINDOW, 0)]
+    Nk = 3 * Nc
+    bf = lambda a: synth.bf16_round(a.astype(np.float32))  # noqa: E731
+    Q = g.standard_normal((1, Nc, 1, 128)) * 0.5
+    Kc = g.standard_normal((1, Nk, 1, 128)) * 0.5
+    Vc = g.standard_normal((1, Nk, 1, 128))
+    if far_logit:
+        # far keys aligned with every query: logit ~ far_logit before the bias
+        Q[..., 0] = math.sqrt(far_logit * math.sqrt(128))
+        Kc[:, Nc + 128:2 * Nc, :, 0] = math.sqrt(far_logit * math.sqrt(128))
+    Q, Kc, Vc = bf(Q), bf(Kc), bf(Vc)
+    p = np.arange(Nc)
+    uv = np.stack([(p % w) * 0.9, (p // w) * (9.0 / (h - 1))], -1)[:, None, :].astype(np.float32)
+    valid = np.ones((Nc, 1), bool)
+    if invalid_row is not None:
+        valid[invalid_row] = False
+    shp = api.shape(1, 1, 128, F, h, w, torch.bfloat16)
+    return shp, Q, Kc, Vc, segs, uv, valid, (F, h, w, k)
+
+
+def test_skip_far_matches_exact_oracle():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _skip_case(30)
+    Os, ls = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, 1, 2.0, 1.0, flags=api.ATTN_SKIP_FAR)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0)
+    _check_bf16(Os, ls, Oo, lo)
+
+
+def test_skip_far_is_active_and_only_an_approximation():
+    # keys so well aligned with the queries that their weights dominate even after the bias:
+    # the exact result is pulled towards them, the skipping kernel never sees them
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _skip_case(31, far_logit=60.0)
+    Oe, _ = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, 1, 2.0, 1.0)
+    Os, _ = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, 1, 2.0, 1.0, flags=api.ATTN_SKIP_FAR)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0)
+    Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, 2.0, 1.0)
+    _check_bf16_peaky(Oe, Oo, Oabs)
+    assert np.abs(Os - Oo).max() > 0.3
+
+
+def test_skip_far_needs_every_query_valid():
+    # one query without a valid correspondence in the frame: nothing is skipped, bit for bit
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _skip_case(32, far_logit=60.0, invalid_row=77)
+    Oe, le = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, 1, 2.0, 1.0)
+    Os, ls = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, 1, 2.0, 1.0, flags=api.ATTN_SKIP_FAR)
+    np.testing.assert_array_equal(Oe, Os)
+    np.testing.assert_array_equal(le, ls)
