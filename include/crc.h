@@ -265,7 +265,8 @@ crc_status crc_gather(const crc_shape* shape, const void* pool, int32_t num_slab
  *           d_idx[r] >= 0, and r < *d_count when d_count is not NULL
  *           (a window-extension slot is not a retrieval and gets no bias).
  * Source frames and depths are read from the bank at chunk d_idx[r] on the device.
- * The per-pair transform is composed in fp64; per-token arithmetic is fp32.
+ * The per-(frame, source frame) transform is composed in fp32 from the fp64 records
+ * (camera-centre difference in fp64); per-token arithmetic is fp32.
  *
  *   cur      host [F] frames of the current chunk;  d_depth [F][h][w] fp32.
  *   d_uv     device [N_q][S][2] fp32 u^ (NaN where undefined), S = k*F.

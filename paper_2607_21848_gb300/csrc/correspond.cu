@@ -5,9 +5,12 @@
 // that every output array is written fully coalesced.  At block start the
 // per-(target frame t, source frame s) transform
 //     A_ts = R_s^T R_t K_t^-1,   b_ts = R_s^T (c_t - c_s),   K_s
-// is composed in fp64 from the current frames (kernel argument) and the bank
-// records of the retrieved chunk d_idx[r] (device memory, so no host round trip)
-// and kept in shared memory as fp32.  Per pair:
+// is composed from the current frames (kernel argument) and the bank records of
+// the retrieved chunk d_idx[r] (device memory, so no host round trip) and kept in
+// shared memory.  The composition runs in fp32 -- the per-pair arithmetic that
+// consumes it is fp32 anyway -- except for the camera-centre difference, which is
+// formed in fp64 so that nearby centres do not cancel; fp64 throughput on this GPU
+// is a small fraction of fp32's and every block repeats the composition.  Per pair:
 //     X_s = z_p A_ts (j, i, 1)^T + b_ts  (= Eq. 3's X_s),   u^ = pi(K_s X_s).
 #include <math.h>
 
@@ -20,19 +23,21 @@ namespace {
 constexpr int kMaxS = CRC_MAX_K * CRC_MAX_FRAMES;
 constexpr int kMaxPairs = CRC_MAX_FRAMES * kMaxS;
 
-struct PairXf {
+// 24 words, 16-byte aligned, so that a pair's transform is six vector loads
+struct __align__(16) PairXf {
   float A[9];
   float b[3];
   float Ks[9];
   int depth_off;  // offset of D_s in the bank depth array, -1 if the pair is not a retrieval
+  int pad[2];
 };
 
-__device__ void mat3_inverse(const double* m, double* inv) {
-  const double c00 = m[4] * m[8] - m[5] * m[7];
-  const double c01 = m[5] * m[6] - m[3] * m[8];
-  const double c02 = m[3] * m[7] - m[4] * m[6];
-  const double det = m[0] * c00 + m[1] * c01 + m[2] * c02;
-  const double id = 1.0 / det;
+__device__ void mat3_inverse(const float* m, float* inv) {
+  const float c00 = m[4] * m[8] - m[5] * m[7];
+  const float c01 = m[5] * m[6] - m[3] * m[8];
+  const float c02 = m[3] * m[7] - m[4] * m[6];
+  const float det = m[0] * c00 + m[1] * c01 + m[2] * c02;
+  const float id = 1.0f / det;
   inv[0] = c00 * id;
   inv[1] = (m[2] * m[7] - m[1] * m[8]) * id;
   inv[2] = (m[1] * m[5] - m[2] * m[4]) * id;
@@ -58,24 +63,25 @@ __global__ void __launch_bounds__(256) correspond_kernel(const __grid_constant__
     bool ok = (j >= 0) && (j < a.capacity);
     if (a.d_count) ok = ok && (r < *a.d_count);
     PairXf x;
+    x.pad[0] = x.pad[1] = 0;
     if (ok) {
       const double* ft = &a.cur.rec[t][0];
       const double* fs = a.bank_frames + ((size_t)j * a.F + f) * kFrameDoubles;
-      double Ki[9], RK[9], A[9];
-      mat3_inverse(ft, Ki);
-      const double* Rt = ft + 9;
-      const double* Rs = fs + 9;
+      float Kt[9], Rt[9], Rs[9], Ki[9], RK[9];
+      for (int e = 0; e < 9; ++e) {
+        Kt[e] = (float)ft[e];
+        Rt[e] = (float)ft[9 + e];
+        Rs[e] = (float)fs[9 + e];
+      }
+      mat3_inverse(Kt, Ki);
       for (int m = 0; m < 3; ++m)
         for (int n = 0; n < 3; ++n) RK[3 * m + n] = Rt[3 * m + 0] * Ki[n] + Rt[3 * m + 1] * Ki[3 + n] + Rt[3 * m + 2] * Ki[6 + n];
       // A = R_s^T (R_t K_t^-1)
       for (int m = 0; m < 3; ++m)
-        for (int n = 0; n < 3; ++n) A[3 * m + n] = Rs[m] * RK[n] + Rs[3 + m] * RK[3 + n] + Rs[6 + m] * RK[6 + n];
-      const double dc[3] = {ft[18] - fs[18], ft[19] - fs[19], ft[20] - fs[20]};
-      for (int m = 0; m < 3; ++m) x.b[m] = (float)(Rs[m] * dc[0] + Rs[3 + m] * dc[1] + Rs[6 + m] * dc[2]);
-      for (int e = 0; e < 9; ++e) {
-        x.A[e] = (float)A[e];
-        x.Ks[e] = (float)fs[e];
-      }
+        for (int n = 0; n < 3; ++n) x.A[3 * m + n] = Rs[m] * RK[n] + Rs[3 + m] * RK[3 + n] + Rs[6 + m] * RK[6 + n];
+      const float dc[3] = {(float)(ft[18] - fs[18]), (float)(ft[19] - fs[19]), (float)(ft[20] - fs[20])};
+      for (int m = 0; m < 3; ++m) x.b[m] = Rs[m] * dc[0] + Rs[3 + m] * dc[1] + Rs[6 + m] * dc[2];
+      for (int e = 0; e < 9; ++e) x.Ks[e] = (float)fs[e];
       x.depth_off = (int)(((size_t)j * a.F + f) * hw);
     } else {
       for (int e = 0; e < 9; ++e) x.A[e] = x.Ks[e] = 0.f;
@@ -89,51 +95,94 @@ __global__ void __launch_bounds__(256) correspond_kernel(const __grid_constant__
   const int total = a.F * hw * S;
   const bool vis_test = !isinf(a.eps);
   const float one_eps = 1.0f + a.eps;
-  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < total; idx += gridDim.x * blockDim.x) {
-    const int p = idx / S;
-    const int s = idx - p * S;
-    const int t = p / hw;
-    const int rem = p - t * hw;
-    const int i = rem / a.w;
-    const int jx = rem - i * a.w;
-    const PairXf& x = px[t * S + s];
-    float ux = __int_as_float(0x7fc00000), uy = ux;  // NaN when the pair is not a retrieval
-    bool valid = false;
-    int cell = -1;
-    if (x.depth_off >= 0) {
-      const float z = a.depth[p];
-      const float u0 = (float)jx, u1 = (float)i;
+  // Each thread carries kILP pairs at once (stride = the whole grid), so that their
+  // query-depth loads and then their source-depth gathers overlap in flight.
+  constexpr int kILP = 4;
+  const int stride = gridDim.x * blockDim.x;
+  for (int base = blockIdx.x * blockDim.x + threadIdx.x; base < total; base += kILP * stride) {
+    int pr[kILP], sr[kILP], jx[kILP], iy[kILP];
+    float z[kILP];
+#pragma unroll
+    for (int u = 0; u < kILP; ++u) {
+      const int idx = base + u * stride;
+      pr[u] = idx < total ? (int)fastdiv((uint32_t)idx, a.div_S) : -1;
+      if (pr[u] >= 0) {
+        sr[u] = idx - pr[u] * S;
+        const int t = (int)fastdiv((uint32_t)pr[u], a.div_hw);
+        const int rem = pr[u] - t * hw;
+        iy[u] = (int)fastdiv((uint32_t)rem, a.div_w);
+        jx[u] = rem - iy[u] * a.w;
+        sr[u] += t * S;  // index of the (t, s) transform
+        z[u] = px[sr[u]].depth_off >= 0 ? a.depth[pr[u]] : 0.f;
+      }
+    }
+    float ux[kILP], uy[kILP], X2[kILP];
+    int cell[kILP];
+    bool valid[kILP];
+#pragma unroll
+    for (int u = 0; u < kILP; ++u) {
+      ux[u] = uy[u] = __int_as_float(0x7fc00000);  // NaN when the pair is not a retrieval
+      valid[u] = false;
+      cell[u] = -1;
+      X2[u] = 0.f;
+      if (pr[u] < 0) continue;
+      PairXf x;
+#pragma unroll
+      for (int v = 0; v < 6; ++v)
+        reinterpret_cast<float4*>(&x)[v] = reinterpret_cast<const float4*>(&px[sr[u]])[v];
+      if (x.depth_off < 0) continue;
+      const float u0 = (float)jx[u], u1 = (float)iy[u];
       const float a0 = x.A[0] * u0 + x.A[1] * u1 + x.A[2];
       const float a1 = x.A[3] * u0 + x.A[4] * u1 + x.A[5];
       const float a2 = x.A[6] * u0 + x.A[7] * u1 + x.A[8];
-      const float X0 = z * a0 + x.b[0];
-      const float X1 = z * a1 + x.b[1];
-      const float X2 = z * a2 + x.b[2];
-      const float q0 = x.Ks[0] * X0 + x.Ks[1] * X1 + x.Ks[2] * X2;
-      const float q1 = x.Ks[3] * X0 + x.Ks[4] * X1 + x.Ks[5] * X2;
-      const float q2 = x.Ks[6] * X0 + x.Ks[7] * X1 + x.Ks[8] * X2;
-      ux = q0 / q2;
-      uy = q1 / q2;
-      const float fx = floorf(ux + 0.5f), fy = floorf(uy + 0.5f);
-      valid = isfinite(z) && z > 0.f && isfinite(ux) && isfinite(uy) && X2 > 0.f && fx >= 0.f &&
-              fx < (float)a.w && fy >= 0.f && fy < (float)a.h;
-      if (valid) {
-        const int cx = (int)fx, cy = (int)fy;
-        if (vis_test) valid = X2 <= one_eps * a.bank_depth[x.depth_off + cy * a.w + cx];
-        if (valid) cell = cy * a.w + cx;
-      }
+      const float X0 = z[u] * a0 + x.b[0];
+      const float X1 = z[u] * a1 + x.b[1];
+      X2[u] = z[u] * a2 + x.b[2];
+      const float q0 = x.Ks[0] * X0 + x.Ks[1] * X1 + x.Ks[2] * X2[u];
+      const float q1 = x.Ks[3] * X0 + x.Ks[4] * X1 + x.Ks[5] * X2[u];
+      const float q2 = x.Ks[6] * X0 + x.Ks[7] * X1 + x.Ks[8] * X2[u];
+      const float iq = 1.0f / q2;  // one division: u^ within an ulp of q0 / q2
+      ux[u] = q0 * iq;
+      uy[u] = q1 * iq;
+      const float fx = floorf(ux[u] + 0.5f), fy = floorf(uy[u] + 0.5f);
+      valid[u] = isfinite(z[u]) && z[u] > 0.f && isfinite(ux[u]) && isfinite(uy[u]) && X2[u] > 0.f && fx >= 0.f &&
+                 fx < (float)a.w && fy >= 0.f && fy < (float)a.h;
+      if (valid[u]) cell[u] = (int)fy * a.w + (int)fx;
     }
-    reinterpret_cast<float2*>(a.uv)[idx] = make_float2(ux, uy);
-    if (a.cell) a.cell[idx] = cell;
-    a.valid[idx] = valid ? 1 : 0;
+    float ds[kILP];
+#pragma unroll
+    for (int u = 0; u < kILP; ++u)
+      ds[u] = (vis_test && valid[u]) ? a.bank_depth[px[sr[u]].depth_off + cell[u]] : 0.f;
+#pragma unroll
+    for (int u = 0; u < kILP; ++u) {
+      if (pr[u] < 0) continue;
+      if (vis_test && valid[u] && !(X2[u] <= one_eps * ds[u])) {
+        valid[u] = false;
+        cell[u] = -1;
+      }
+      const int idx = base + u * stride;
+      reinterpret_cast<float2*>(a.uv)[idx] = make_float2(ux[u], uy[u]);
+      if (a.cell) a.cell[idx] = cell[u];
+      a.valid[idx] = valid[u] ? 1 : 0;
+    }
   }
 }
 
 cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s) {
   const int total = a.F * a.h * a.w * a.k * a.F;
   if (total == 0) return cudaSuccess;
-  int blocks = (total + 255) / 256;
-  if (blocks > 4096) blocks = 4096;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // grid-stride over the pairs with four pairs in flight per thread: one resident
+  // wave, so that each block's composition of the transforms is amortised over
+  // many pairs
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel, 256, 0) != cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  int blocks = (total + 1023) / 1024;
+  if (blocks > per_sm * sms) blocks = per_sm * sms;
   correspond_kernel<<<blocks, 256, 0, s>>>(a);
   return cudaGetLastError();
 }

@@ -43,7 +43,7 @@ CONFIG_NAMES = {
     5: "wan1.3b_loop_stream_k2",
 }
 
-_PURPOSES = ("poses", "depth", "q", "k", "v", "bank", "scene", "pool", "step")
+_PURPOSES = ("poses", "depth", "q", "k", "v", "bank", "scene", "pool", "step", "sweep")
 
 
 def rng(seed: int, purpose: str, *extra: int) -> np.random.Generator:
