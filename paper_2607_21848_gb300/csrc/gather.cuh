@@ -99,6 +99,11 @@ struct Vec16<false> {
 // (channel0 is even).  Half-split pairs (c, c + pairs) lie in two vectors `half`
 // apart (channel0 and pairs are multiples of the vector width); the lane that
 // owns the lower vector rotates and writes both.  Four vectors per lane in flight.
+//
+// When the vectors of a head divide the warp (d / N in {1, 2, 4, 8, 16, 32}), lane l
+// meets the same channels (l mod d/N) * N in every head it copies, so its kind of
+// vector and its (cos, sin) factors are fixed for the whole row: taken once, in
+// registers.  Other head sizes take the general per-vector path.
 template <bool BF16>
 __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict__ dst, const GatherArgs& g,
                                  const float2* __restrict__ cs, int lane) {
@@ -110,53 +115,86 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
   const int vph = g.d / N;  // vectors per head
   const int c0 = g.rope_c0, np = g.rope_pairs, np2 = 2 * g.rope_pairs;
   const int half = np / N;
-  for (int base = lane; base < n; base += 128) {
-    uint4 v[4], w[4];
-    int kind[4], ch[4];
+  if ((32 % vph) == 0) {
+    const int ch = (lane % vph) * N;
+    const int kind = g.rope_interleaved ? ((ch + N > c0 && ch < c0 + np2) ? 1 : 0)
+                                        : ((ch >= c0 && ch < c0 + np) ? 2 : ((ch >= c0 + np && ch < c0 + np2) ? 3 : 0));
+    if (kind == 3) return;  // the lane owning the lower half writes this vector
+    float2 f[N];            // (cos, sin) of each element's pair; (1, 0) outside the block
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int c = base + 32 * u;
-      kind[u] = -1;  // past the row
-      ch[u] = 0;
-      if (c < n) {
-        ch[u] = (c % vph) * N;
-        if (g.rope_interleaved)
-          kind[u] = (ch[u] + N > c0 && ch[u] < c0 + np2) ? 1 : 0;
-        else
-          kind[u] = (ch[u] >= c0 && ch[u] < c0 + np) ? 2 : ((ch[u] >= c0 + np && ch[u] < c0 + np2) ? 3 : 0);
-        if (kind[u] != 3) v[u] = __ldg(s + c);
-        if (kind[u] == 2) w[u] = __ldg(s + c + half);
+    for (int e = 0; e < N; ++e) {
+      const int i = kind == 1 ? (ch + e - c0) >> 1 : ch - c0 + e;
+      const bool in = kind == 1 ? (ch + e >= c0 && ch + e < c0 + np2) : (kind == 2);
+      f[e] = in ? cs[i] : make_float2(1.f, 0.f);
+    }
+    for (int base = lane; base < n; base += 64) {
+      uint4 v[2], w[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int c = base + 32 * u;
+        if (c < n) {
+          v[u] = __ldg(s + c);
+          if (kind == 2) w[u] = __ldg(s + c + half);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int c = base + 32 * u;
+        if (c >= n) break;
+        if (kind == 0) {
+          d[c] = v[u];
+        } else if (kind == 1) {
+          float x[N];
+          IO::unpack(v[u], x);
+#pragma unroll
+          for (int e = 0; e < N; e += 2) rotate_pair(x[e], x[e + 1], f[e]);
+          d[c] = IO::pack(x);
+        } else {
+          float x[N], y[N];
+          IO::unpack(v[u], x);
+          IO::unpack(w[u], y);
+#pragma unroll
+          for (int e = 0; e < N; ++e) rotate_pair(x[e], y[e], f[e]);
+          d[c] = IO::pack(x);
+          d[c + half] = IO::pack(y);
+        }
       }
     }
+    return;
+  }
+  for (int c = lane; c < n; c += 32) {
+    const int ch = (c % vph) * N;
+    const int kind = g.rope_interleaved
+                         ? ((ch + N > c0 && ch < c0 + np2) ? 1 : 0)
+                         : ((ch >= c0 && ch < c0 + np) ? 2 : ((ch >= c0 + np && ch < c0 + np2) ? 3 : 0));
+    if (kind == 0) {
+      d[c] = __ldg(s + c);
+    } else if (kind == 1) {
+      float x[N];
+      IO::unpack(__ldg(s + c), x);
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int c = base + 32 * u;
-      if (kind[u] == 0) {
-        d[c] = v[u];
-      } else if (kind[u] == 1) {
-        float x[N];
-        IO::unpack(v[u], x);
-#pragma unroll
-        for (int e = 0; e < N; e += 2) {
-          const int che = ch[u] + e;
-          if (che >= c0 && che < c0 + np2) rotate_pair(x[e], x[e + 1], cs[(che - c0) >> 1]);
-        }
-        d[c] = IO::pack(x);
-      } else if (kind[u] == 2) {
-        float x[N], y[N];
-        IO::unpack(v[u], x);
-        IO::unpack(w[u], y);
-#pragma unroll
-        for (int e = 0; e < N; ++e) rotate_pair(x[e], y[e], cs[ch[u] - c0 + e]);
-        d[c] = IO::pack(x);
-        d[c + half] = IO::pack(y);
+      for (int e = 0; e < N; e += 2) {
+        const int che = ch + e;
+        if (che >= c0 && che < c0 + np2) rotate_pair(x[e], x[e + 1], cs[(che - c0) >> 1]);
       }
+      d[c] = IO::pack(x);
+    } else if (kind == 2) {
+      float x[N], y[N];
+      IO::unpack(__ldg(s + c), x);
+      IO::unpack(__ldg(s + c + half), y);
+#pragma unroll
+      for (int e = 0; e < N; ++e) rotate_pair(x[e], y[e], cs[ch - c0 + e]);
+      d[c] = IO::pack(x);
+      d[c + half] = IO::pack(y);
     }
   }
 }
 
 // Copies every active slot's K and V rows (one warp per token row, rows ordered
 // (active slot, K|V, layer, token)) from its slab into the slot's cache segment.
+// ROPE = false compiles the plain copy only (no re-positioning requested), which
+// keeps the register footprint, and so the copy's occupancy, of a plain gather.
+template <bool ROPE>
 __device__ inline void gather_slots(const GatherArgs& g, int k, const GatherPlan& p) {
   int act[CRC_MAX_K];
   int n_act = 0;
@@ -179,7 +217,7 @@ __device__ inline void gather_slots(const GatherArgs& g, int k, const GatherPlan
     const char* src = g.pool + slab * g.slab_bytes + kv * g.kv_bytes + rem * g.row_bytes;
     char* dst = (kv ? g.cache_v : g.cache_k) + l * g.cache_layer_stride +
                 (int64_t)(g.slot_offset[r] + t) * g.cache_token_stride;
-    if (kv == 0 && p.rotate[r]) {
+    if (ROPE && kv == 0 && p.rotate[r]) {
       if (g.elem_bytes == 2)
         copy_row_rotated<true>(src, dst, g, p.cs[r], lane);
       else

@@ -43,7 +43,8 @@ __device__ __forceinline__ void score_entry(const double* __restrict__ centre, c
 
 }  // namespace
 
-__global__ void __launch_bounds__(256) retrieve_gather_kernel(const __grid_constant__ RetrieveArgs a) {
+template <bool ROPE>
+__global__ void __launch_bounds__(256, ROPE ? 2 : 4) retrieve_gather_kernel(const __grid_constant__ RetrieveArgs a) {
   __shared__ double sh_cn[3], sh_vn[3];
   __shared__ double red_s[8];
   __shared__ int red_j[8];
@@ -134,17 +135,18 @@ __global__ void __launch_bounds__(256) retrieve_gather_kernel(const __grid_const
   }
   __syncthreads();
   if (a.g.pool == nullptr) return;
-  plan_rope(a.g, a.k, plan);
-  gather_slots(a.g, a.k, plan);
+  if (ROPE) plan_rope(a.g, a.k, plan);
+  gather_slots<ROPE>(a.g, a.k, plan);
 }
 
 // The gather alone, for a cache that mirrors the retrieved slots of a step.
-__global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherOnlyArgs a) {
+template <bool ROPE>
+__global__ void __launch_bounds__(256, ROPE ? 2 : 4) gather_kernel(const __grid_constant__ GatherOnlyArgs a) {
   __shared__ GatherPlan plan;
   if (threadIdx.x < a.k) plan.chunk[threadIdx.x] = a.d_idx[threadIdx.x];
   __syncthreads();
-  plan_rope(a.g, a.k, plan);
-  gather_slots(a.g, a.k, plan);
+  if (ROPE) plan_rope(a.g, a.k, plan);
+  gather_slots<ROPE>(a.g, a.k, plan);
 }
 
 namespace {
@@ -164,12 +166,18 @@ int gather_blocks(int k, const GatherArgs& g) {
 
 cudaError_t launch_retrieve(const RetrieveArgs& a, cudaStream_t s) {
   const int blocks = a.g.pool ? gather_blocks(a.k, a.g) : 1;
-  retrieve_gather_kernel<<<blocks, 256, 0, s>>>(a);
+  if (a.g.pool && a.g.rope_pairs > 0)
+    retrieve_gather_kernel<true><<<blocks, 256, 0, s>>>(a);
+  else
+    retrieve_gather_kernel<false><<<blocks, 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 
 cudaError_t launch_gather(const GatherOnlyArgs& a, cudaStream_t s) {
-  gather_kernel<<<gather_blocks(a.k, a.g), 256, 0, s>>>(a);
+  if (a.g.rope_pairs > 0)
+    gather_kernel<true><<<gather_blocks(a.k, a.g), 256, 0, s>>>(a);
+  else
+    gather_kernel<false><<<gather_blocks(a.k, a.g), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 

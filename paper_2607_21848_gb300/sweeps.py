@@ -1,10 +1,47 @@
-"""Stand-alone sweeps of single kernels at scales larger than the chunk step, for
-profiling (e.g. under ncu): `python -m paper_2607_21848_gb300.sweeps correspond`."""
+"""Stand-alone sweeps of single kernels, for measurement and profiling (e.g. under ncu):
+
+  python -m paper_2607_21848_gb300.sweeps correspond   # 126 MB reprojection sweep
+  python -m paper_2607_21848_gb300.sweeps gather       # crc_gather, plain and re-positioned
+"""
 
 from __future__ import annotations
 
 import json
 import sys
+
+
+def gather_sweep(device="cuda:0", iters: int = 10):
+    """crc_gather of one retrieved chunk at the Wan-1.3B chunk shape (30 layers, 12 heads,
+    d = 128, 4680 tokens), plain and with the keys re-positioned (22 interleaved temporal
+    rotary pairs): 862.6 MB read and 862.6 MB written per call either way."""
+    import torch
+
+    import synth
+    from paper_2607_21848_gb300 import api
+
+    wl = synth.make_workload(2, layers=30)
+    L, Nc, H, d = wl.L, wl.Nc, wl.H, wl.d
+    g = torch.Generator(device=device).manual_seed(3)
+    pool = (torch.randn(2, 2, L, Nc, H, d, generator=g, device=device) * wl.qkv_scale).to(torch.bfloat16)
+    segs = [(0, Nc, api.SEG_SINK, 0), (Nc, Nc, api.SEG_RETRIEVED, 0), (2 * Nc, 2 * Nc, api.SEG_WINDOW, 0)]
+    cache = api.Cache.empty(L, 4 * Nc, H, d, torch.bfloat16, segs, device=device)
+    shp = api.shape(L, H, d, wl.F, wl.h, wl.w, torch.bfloat16)
+    idx = torch.tensor([33], dtype=torch.int32, device=device)
+    out = {}
+    for name, rope in (("plain", None), ("rope", api.rope_params(0, 22, 10000.0, True, pos_slot0=189, pos_stride=3))):
+        api.crc_gather(shp, pool, idx, 1, cache, rope=rope)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(iters):
+            api.crc_gather(shp, pool, idx, 1, cache, rope=rope)
+        e1.record()
+        torch.cuda.synchronize()
+        t = e0.elapsed_time(e1) / 1e3 / iters
+        nbytes = 2 * 2 * L * Nc * H * d * 2
+        out[name] = {"bytes": nbytes, "ms": t * 1e3, "gbs": nbytes / t / 1e9}
+    return out
 
 
 def main(argv=None):
@@ -19,6 +56,8 @@ def main(argv=None):
     build.build()
     if what == "correspond":
         print(json.dumps(bench.correspond_sweep("cuda:0")))
+    elif what == "gather":
+        print(json.dumps(gather_sweep("cuda:0")))
     else:
         raise SystemExit(f"unknown sweep {what}")
 
