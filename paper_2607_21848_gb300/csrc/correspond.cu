@@ -95,29 +95,36 @@ __global__ void __launch_bounds__(256) correspond_kernel(const __grid_constant__
   const int total = a.F * hw * S;
   const bool vis_test = !isinf(a.eps);
   const float one_eps = 1.0f + a.eps;
-  // Each thread carries kILP pairs at once (stride = the whole grid), so that their
-  // query-depth loads and then their source-depth gathers overlap in flight.
+  // The block size is a multiple of S, so the grid stride is too and each thread
+  // keeps one source frame s for all its pairs.  Its transform for target frame t
+  // stays in registers and is reloaded only when t changes (at most F times).
+  // Each thread carries kILP pairs at once, so that their query-depth loads and
+  // then their source-depth gathers overlap in flight.
   constexpr int kILP = 4;
   const int stride = gridDim.x * blockDim.x;
-  for (int base = blockIdx.x * blockDim.x + threadIdx.x; base < total; base += kILP * stride) {
-    int pr[kILP], sr[kILP], jx[kILP], iy[kILP];
+  const int first = blockIdx.x * blockDim.x + threadIdx.x;
+  const int s_own = first - (int)fastdiv((uint32_t)first, a.div_S) * S;
+  int t_cached = -1;
+  PairXf x;
+  for (int base = first; base < total; base += kILP * stride) {
+    int pr[kILP], tr[kILP], jx[kILP], iy[kILP];
     float z[kILP];
 #pragma unroll
     for (int u = 0; u < kILP; ++u) {
       const int idx = base + u * stride;
       pr[u] = idx < total ? (int)fastdiv((uint32_t)idx, a.div_S) : -1;
+      tr[u] = -1;
+      z[u] = 0.f;
       if (pr[u] >= 0) {
-        sr[u] = idx - pr[u] * S;
-        const int t = (int)fastdiv((uint32_t)pr[u], a.div_hw);
-        const int rem = pr[u] - t * hw;
+        tr[u] = (int)fastdiv((uint32_t)pr[u], a.div_hw);
+        const int rem = pr[u] - tr[u] * hw;
         iy[u] = (int)fastdiv((uint32_t)rem, a.div_w);
         jx[u] = rem - iy[u] * a.w;
-        sr[u] += t * S;  // index of the (t, s) transform
-        z[u] = px[sr[u]].depth_off >= 0 ? a.depth[pr[u]] : 0.f;
+        z[u] = a.depth[pr[u]];
       }
     }
     float ux[kILP], uy[kILP], X2[kILP];
-    int cell[kILP];
+    int cell[kILP], doff[kILP];
     bool valid[kILP];
 #pragma unroll
     for (int u = 0; u < kILP; ++u) {
@@ -125,11 +132,15 @@ __global__ void __launch_bounds__(256) correspond_kernel(const __grid_constant__
       valid[u] = false;
       cell[u] = -1;
       X2[u] = 0.f;
+      doff[u] = -1;
       if (pr[u] < 0) continue;
-      PairXf x;
+      if (tr[u] != t_cached) {
 #pragma unroll
-      for (int v = 0; v < 6; ++v)
-        reinterpret_cast<float4*>(&x)[v] = reinterpret_cast<const float4*>(&px[sr[u]])[v];
+        for (int v = 0; v < 6; ++v)
+          reinterpret_cast<float4*>(&x)[v] = reinterpret_cast<const float4*>(&px[tr[u] * S + s_own])[v];
+        t_cached = tr[u];
+      }
+      doff[u] = x.depth_off;
       if (x.depth_off < 0) continue;
       const float u0 = (float)jx[u], u1 = (float)iy[u];
       const float a0 = x.A[0] * u0 + x.A[1] * u1 + x.A[2];
@@ -152,7 +163,7 @@ __global__ void __launch_bounds__(256) correspond_kernel(const __grid_constant__
     float ds[kILP];
 #pragma unroll
     for (int u = 0; u < kILP; ++u)
-      ds[u] = (vis_test && valid[u]) ? a.bank_depth[px[sr[u]].depth_off + cell[u]] : 0.f;
+      ds[u] = (vis_test && valid[u]) ? a.bank_depth[doff[u] + cell[u]] : 0.f;
 #pragma unroll
     for (int u = 0; u < kILP; ++u) {
       if (pr[u] < 0) continue;
@@ -177,13 +188,15 @@ cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s) {
   // grid-stride over the pairs with four pairs in flight per thread: one resident
   // wave, so that each block's composition of the transforms is amortised over
   // many pairs
+  const int S = a.k * a.F;
+  const int threads = (256 / S) * S;  // a multiple of S (S <= 32)
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel, 256, 0) != cudaSuccess ||
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel, threads, 0) != cudaSuccess ||
       per_sm < 1)
     per_sm = 1;
-  int blocks = (total + 1023) / 1024;
+  int blocks = (total + 4 * threads - 1) / (4 * threads);
   if (blocks > per_sm * sms) blocks = per_sm * sms;
-  correspond_kernel<<<blocks, 256, 0, s>>>(a);
+  correspond_kernel<<<blocks, threads, 0, s>>>(a);
   return cudaGetLastError();
 }
 
