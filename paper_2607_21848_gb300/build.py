@@ -34,8 +34,20 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
+def _flags():
+    """Compile flags; CRC_NVTX=1 in the environment adds NVTX ranges to the entry points."""
+    extra = ["-DCRC_NVTX"] if os.environ.get("CRC_NVTX") == "1" else []
+    return FLAGS + extra
+
+
 def build(verbose: bool = False, force: bool = False) -> str:
     os.makedirs(BUILD, exist_ok=True)
+    flags = _flags()
+    stamp = os.path.join(BUILD, "flags.txt")
+    if not os.path.exists(stamp) or open(stamp).read() != " ".join(flags):
+        force = True  # objects built with other flags
+        with open(stamp, "w") as f:
+            f.write(" ".join(flags))
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))]
     headers.append(os.path.join(INCLUDE, "crc.h"))
     cc = nvcc()
@@ -46,7 +58,7 @@ def build(verbose: bool = False, force: bool = False) -> str:
         o = os.path.join(BUILD, src.replace(".cu", ".o"))
         objs.append(o)
         if force or _stale(o, [s] + headers):
-            jobs.append([cc, *ARCH, *FLAGS, "-c", s, "-o", o])
+            jobs.append([cc, *ARCH, *flags, "-c", s, "-o", o])
 
     def run(cmd):
         r = subprocess.run(cmd, capture_output=True, text=True)

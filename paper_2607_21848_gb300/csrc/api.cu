@@ -4,6 +4,23 @@
 
 #include "internal.cuh"
 
+// Build with -DCRC_NVTX (CRC_NVTX=1 in the environment of the build script) to wrap
+// every entry point in an NVTX range, for timeline tools.
+#ifdef CRC_NVTX
+#include <nvtx3/nvToolsExt.h>
+namespace {
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
+}  // namespace
+#define CRC_RANGE(name) NvtxRange crc_nvtx_range_(name)
+#else
+#define CRC_RANGE(name) \
+  do {                  \
+  } while (0)
+#endif
+
 namespace {
 
 thread_local int32_t g_last_cuda_error = 0;
@@ -168,6 +185,7 @@ int32_t crc_last_cuda_error(void) { return g_last_cuda_error; }
 
 crc_status crc_bank_insert_poses(const crc_bank* bank, const crc_shape* shape, int32_t first, int32_t count,
                                  const crc_frame* frames, cudaStream_t s) {
+  CRC_RANGE("crc_bank_insert_poses");
   crc_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_bank(bank, false))) return st;
@@ -189,6 +207,7 @@ crc_status crc_bank_insert_poses(const crc_bank* bank, const crc_shape* shape, i
 crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_t chunk, const crc_frame* frames,
                             const float* d_depth, const void* d_k, const void* d_v, const crc_cache* cache,
                             int32_t window_offset, cudaStream_t s) {
+  CRC_RANGE("crc_cache_update");
   crc_status st = check_shape(shape);
   if (st) return st;
   const bool with_kv = d_k != nullptr || d_v != nullptr;
@@ -235,6 +254,7 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
 crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
                         int32_t n, const crc_retrieval* p, const crc_cache* cache, const crc_rope* rope,
                         int32_t* d_idx, double* d_score, int32_t* d_count, cudaStream_t s) {
+  CRC_RANGE("crc_retrieve");
   crc_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_bank(bank, cache != nullptr))) return st;
@@ -271,6 +291,7 @@ crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shap
 
 crc_status crc_gather(const crc_shape* shape, const void* pool, int32_t num_slabs, const int32_t* d_idx, int32_t k,
                       const crc_cache* cache, const crc_rope* rope, cudaStream_t s) {
+  CRC_RANGE("crc_gather");
   crc_status st = check_shape(shape);
   if (st) return st;
   if (!d_idx || !cache || k < 1 || k > CRC_MAX_K) return CRC_ERR_INVALID_ARG;
@@ -286,6 +307,7 @@ crc_status crc_gather(const crc_shape* shape, const void* pool, int32_t num_slab
 crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const float* d_depth, const crc_bank* bank,
                           const int32_t* d_idx, const int32_t* d_count, int32_t k, float eps, float* d_uv,
                           int32_t* d_cell, uint8_t* d_valid, cudaStream_t s) {
+  CRC_RANGE("crc_correspond");
   crc_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_bank(bank, false))) return st;
@@ -321,6 +343,7 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
                                 float* d_lse, int32_t n_q, const float* d_uv, const uint8_t* d_valid, int32_t k,
                                 const int32_t* d_slot_chunk, float lambda, float sigma, int32_t flags,
                                 int32_t* d_status, cudaStream_t s) {
+  CRC_RANGE("crc_biased_attention");
   crc_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_cache(cache, shape))) return st;

@@ -98,6 +98,29 @@ class ChunkStream:
                                          device=device)
             self.control_cache = api.Cache.empty(c.control_L, c.n_keys, c.H, c.d, c.dtype, [], device=device)
 
+    # ---- checkpoint -------------------------------------------------------
+    def state_dict(self) -> dict:
+        """Everything a later step reads: the bank (poses, pose summaries, depth, K/V
+        slabs), the cache and, if present, the control branch's pool and cache.  The
+        step index is the caller's (segments and ring slots follow from it).  The
+        tensors are the stream's own; save or clone them before stepping on."""
+        sd = {"bank." + k: getattr(self.bank, k) for k in ("frames", "centre", "view", "depth", "kv")}
+        sd["cache.k"], sd["cache.v"] = self.cache.k, self.cache.v
+        if self.control_shape is not None:
+            sd["control_bank.kv"] = self.control_bank.kv
+            sd["control_cache.k"], sd["control_cache.v"] = self.control_cache.k, self.control_cache.v
+        return sd
+
+    def load_state_dict(self, sd: dict) -> None:
+        """Restore a state_dict() of a stream with the same configuration."""
+        own = self.state_dict()
+        if set(own) != set(sd):
+            raise ValueError(f"state keys differ: {sorted(set(own) ^ set(sd))}")
+        for k, t in own.items():
+            if tuple(t.shape) != tuple(sd[k].shape) or t.dtype != sd[k].dtype:
+                raise ValueError(f"{k}: expected {tuple(t.shape)} {t.dtype}")
+            t.copy_(sd[k])
+
     # ---- layout -----------------------------------------------------------
     def slot_offset(self, r: int) -> int:
         return (1 + r) * self.cfg.Nc
