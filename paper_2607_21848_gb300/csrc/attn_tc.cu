@@ -489,20 +489,50 @@ __global__ void __launch_bounds__(kThreads, 1)
         return ti.cls != CLS_AUG ||
                mbar_wait(bar(B_BFULL(ti.q % NBB)), (ti.q / NBB) & 1, abort_flag, T, kHintMma);
       };
+      // query tile 1 may hold no query at all (the last CTA of a head); then only
+      // tile 0's MMAs run, and they release the stages and bias operands
+      const bool live1 = q0 + BM < a.Nq;
       TileInfo t0 = tiles[0];
       bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_KFULL(0)), 0, abort_flag, T) &&
-                mbar_wait(bar(B_AREADY(0)), 0, abort_flag, T) && mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T) &&
-                bias_ready(t0);
+                mbar_wait(bar(B_AREADY(0)), 0, abort_flag, T) &&
+                (!live1 || mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T)) && bias_ready(t0);
       if (!ok) fail(P, abort_flag, 3);
       if (ok) {
         tc_fence_after();
         issue_qk(0, 0, t0);
         mma_commit(bar(B_SFULL(0)));
-        issue_qk(1, 0, t0);
-        mma_commit(bar(B_SFULL(1)));
+        if (live1) {
+          issue_qk(1, 0, t0);
+          mma_commit(bar(B_SFULL(1)));
+        }
         mma_commit(bar(B_KEMPTY(0)));
         if (t0.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(t0.q % NBB)));
-        for (int j = 0; j < nt && ok; ++j) {
+        // tile 0 alone: its MMAs release every stage and bias operand
+        for (int j = 0; j < nt && ok && !live1; ++j) {
+          const int st = j % ST;
+          const int jn = j + 1, stn = jn % ST;
+          const bool more = jn < nt;
+          const TileInfo tn = more ? tiles[jn] : t0;
+          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma) &&
+               mbar_wait(bar(B_VFULL(st)), (j / ST) & 1, abort_flag, T, kHintMma);
+          if (!ok) { fail(P, abort_flag, 4); break; }
+          tc_fence_after();
+          issue_pv(0, st, j > 0);
+          mma_commit(bar(B_VEMPTY(st)));
+          if (more) {
+            ok = mbar_wait(bar(B_KFULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma) && bias_ready(tn);
+            if (!ok) { fail(P, abort_flag, 5); break; }
+            tc_fence_after();
+            issue_qk(0, stn, tn);
+            mma_commit(bar(B_SFULL(0)));
+            mma_commit(bar(B_KEMPTY(stn)));
+            if (tn.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(tn.q % NBB)));
+          } else {
+            mma_commit(bar(B_OFINAL(0)));
+          }
+        }
+        // both tiles, interleaved on the tensor core
+        for (int j = 0; j < nt && ok && live1; ++j) {
           const int st = j % ST;
           const int jn = j + 1, stn = jn % ST;
           const bool more = jn < nt;
@@ -549,6 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int wq = warp & 3;          // TMEM lane quarter
     const int r = wq * 32 + lane;     // row in tile = TMEM lane
     const int p = q0 + x * BM + r;    // query index
+    if (q0 + x * BM < a.Nq) {         // else: a query tile without any query, no MMA runs for it
     const bool row_ok = p < a.Nq;
     const uint32_t trow = tmem + ((uint32_t)(wq * 32) << 16);
     const uint32_t tS = trow + TM_S + 128u * x;
@@ -679,6 +710,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (row_ok && a.lse)
       a.lse[((int64_t)layer * a.H + head) * a.Nq + p] = (l > 0.f) ? (m + log2f(l)) * 0.69314718055994531f : -INFINITY;
+    }
   }
 
   tc_fence_before();
