@@ -30,7 +30,12 @@
 //               128-byte swizzled boxes of 128 rows x 64 elements
 //   warp  9     TMEM owner and single-thread tcgen05.mma issuer
 //   warps 10-11 build, ahead of use, the key-side bias/mask operand of every tile
-//               that needs one (3-deep ring, mbarrier handshake with the MMA warp)
+//               that needs one (3-deep ring; the producer declares a stage full only
+//               once the tile's operand is built, and an MMA commit frees the slot)
+// One FULL barrier per stage stands for K, V and the bias operand together, and one
+// EMPTY barrier (a commit after the tile's last PV) frees the whole stage: the
+// single MMA-issuing thread waits once per KV tile for data, since issuing a
+// 128 x 128 x 16 MMA occupies it for nearly as long as the tensor core runs it.
 // The query-side bias operand of each query tile is written by its own softmax
 // warpgroup whenever the source frame of the next biased tile changes.
 // TMEM (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each.  S = Q K^T is an
@@ -91,7 +96,7 @@ constexpr int OFF_AQ = OFF_V + ST * TILE;      // query-side bias operand, one p
 constexpr int OFF_RB = OFF_AQ + NQT * AUG;     // key-side bias/mask operand ring
 constexpr int OFF_TILES = OFF_RB + NBB * AUG;
 constexpr int OFF_BAR = OFF_TILES + kMaxTiles * 12;
-constexpr int NBAR = 1 + 4 * ST + 3 * NQT + 1 + NQT + 2 * NBB;
+constexpr int NBAR = 1 + 2 * ST + 3 * NQT + 1 + NQT + 2 * NBB;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
 constexpr int OFF_BOX = OFF_MISC + 64;  // per source frame: correspondence box of the CTA's queries
 constexpr int SMEM_BYTES = OFF_BOX + CRC_MAX_K * CRC_MAX_FRAMES * 5 * 4 + 1024;  // + slack for 1024-byte alignment
@@ -122,18 +127,18 @@ struct TcParams {
 };
 
 // barrier indices
+// FULL(s): K, V and (for a biased or ragged tile) the key-side bias/mask operand of
+// stage s are in shared memory.  EMPTY(s): the stage's last MMA (PV of tile 1) retired.
 __device__ __forceinline__ int B_QFULL() { return 0; }
-__device__ __forceinline__ int B_KFULL(int s) { return 1 + s; }
-__device__ __forceinline__ int B_KEMPTY(int s) { return 1 + ST + s; }
-__device__ __forceinline__ int B_VFULL(int s) { return 1 + 2 * ST + s; }
-__device__ __forceinline__ int B_VEMPTY(int s) { return 1 + 3 * ST + s; }
-__device__ __forceinline__ int B_SFULL(int x) { return 1 + 4 * ST + x; }
-__device__ __forceinline__ int B_PREADY(int x) { return 1 + 4 * ST + NQT + x; }
-__device__ __forceinline__ int B_OFINAL(int x) { return 1 + 4 * ST + 2 * NQT + x; }
-__device__ __forceinline__ int B_DRAIN() { return 1 + 4 * ST + 3 * NQT; }
-__device__ __forceinline__ int B_AREADY(int x) { return 2 + 4 * ST + 3 * NQT + x; }
-__device__ __forceinline__ int B_BFULL(int b) { return 2 + 4 * ST + 4 * NQT + b; }
-__device__ __forceinline__ int B_BEMPTY(int b) { return 2 + 4 * ST + 4 * NQT + NBB + b; }
+__device__ __forceinline__ int B_FULL(int s) { return 1 + s; }
+__device__ __forceinline__ int B_EMPTY(int s) { return 1 + ST + s; }
+__device__ __forceinline__ int B_SFULL(int x) { return 1 + 2 * ST + x; }
+__device__ __forceinline__ int B_PREADY(int x) { return 1 + 2 * ST + NQT + x; }
+__device__ __forceinline__ int B_OFINAL(int x) { return 1 + 2 * ST + 2 * NQT + x; }
+__device__ __forceinline__ int B_DRAIN() { return 1 + 2 * ST + 3 * NQT; }
+__device__ __forceinline__ int B_AREADY(int x) { return 2 + 2 * ST + 3 * NQT + x; }
+__device__ __forceinline__ int B_BFULL(int b) { return 2 + 2 * ST + 4 * NQT + b; }
+__device__ __forceinline__ int B_BEMPTY(int b) { return 2 + 2 * ST + 4 * NQT + NBB + b; }
 
 // ---- packed fp32 pairs (Blackwell f32x2 ALU ops) and three-input max ----------
 __device__ __forceinline__ uint64_t pk2(float a, float b) {
@@ -258,10 +263,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     mbar_init(bar(B_QFULL()), 1);
     for (int s = 0; s < ST; ++s) {
-      mbar_init(bar(B_KFULL(s)), 1);
-      mbar_init(bar(B_KEMPTY(s)), 1);
-      mbar_init(bar(B_VFULL(s)), 1);
-      mbar_init(bar(B_VEMPTY(s)), 1);
+      mbar_init(bar(B_FULL(s)), 1);
+      mbar_init(bar(B_EMPTY(s)), 1);
     }
     for (int x = 0; x < NQT; ++x) {
       mbar_init(bar(B_SFULL(x)), 1);
@@ -381,31 +384,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int x = 0; x < NQT; ++x)
         for (int b = 0; b < 2; ++b)
           tma_load_4d(sbase + OFF_Q + x * TILE + b * BOX, &tmQ, bar(B_QFULL()), b * 64, head, q0 + x * BM, layer);
-      int issued_k = 0, issued_v = 0;
+      // one full barrier per stage covers K, V and the tile's bias/mask operand, so
+      // that the MMA issuer waits once per KV tile
+      int issued = 0;
       for (int j = 0; j < nt; ++j) {
         const int st = j % ST;
         const uint32_t par = ((j / ST) & 1) ^ 1;
-        const int key0 = (int)tiles[j].key0;
-        if (!mbar_wait(bar(B_KEMPTY(st)), par, abort_flag, T, kHintLoad)) { fail(P, abort_flag, 1); break; }
-        mbar_arrive_expect_tx(bar(B_KFULL(st)), TILE);
+        const TileInfo ti = tiles[j];
+        if (!mbar_wait(bar(B_EMPTY(st)), par, abort_flag, T, kHintLoad)) {
+          fail(P, abort_flag, 1);
+          break;
+        }
+        if (ti.cls == CLS_AUG &&
+            !mbar_wait(bar(B_BFULL(ti.q % NBB)), (ti.q / NBB) & 1, abort_flag, T, kHintLoad)) {
+          fail(P, abort_flag, 2);
+          break;
+        }
+        mbar_arrive_expect_tx(bar(B_FULL(st)), 2 * TILE);
         for (int b = 0; b < 2; ++b)
-          tma_load_4d(sbase + OFF_K + st * TILE + b * BOX, &tmK, bar(B_KFULL(st)), b * 64, head, key0, layer);
-        issued_k = j + 1;
-        if (!mbar_wait(bar(B_VEMPTY(st)), par, abort_flag, T, kHintLoad)) { fail(P, abort_flag, 2); break; }
-        mbar_arrive_expect_tx(bar(B_VFULL(st)), TILE);
+          tma_load_4d(sbase + OFF_K + st * TILE + b * BOX, &tmK, bar(B_FULL(st)), b * 64, head, (int)ti.key0, layer);
         for (int b = 0; b < 2; ++b)
-          tma_load_4d(sbase + OFF_V + st * TILE + b * BOX, &tmV, bar(B_VFULL(st)), b * 64, head, key0, layer);
-        issued_v = j + 1;
+          tma_load_4d(sbase + OFF_V + st * TILE + b * BOX, &tmV, bar(B_FULL(st)), b * 64, head, (int)ti.key0, layer);
+        issued = j + 1;
       }
       if (*abort_flag) {
         // let the copies already issued land before the CTA can exit
         const uint64_t lim = 100000000ull;
         volatile int never = 0;
         mbar_wait(bar(B_QFULL()), 0, &never, lim);
-        for (int j = (issued_k > ST ? issued_k - ST : 0); j < issued_k; ++j)
-          mbar_wait(bar(B_KFULL(j % ST)), (j / ST) & 1, &never, lim);
-        for (int j = (issued_v > ST ? issued_v - ST : 0); j < issued_v; ++j)
-          mbar_wait(bar(B_VFULL(j % ST)), (j / ST) & 1, &never, lim);
+        for (int j = (issued > ST ? issued - ST : 0); j < issued; ++j)
+          mbar_wait(bar(B_FULL(j % ST)), (j / ST) & 1, &never, lim);
       }
     }
    } else if (warp > kWarpMma) {
@@ -484,18 +492,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < BN / 16; ++kk)
           mma_ts(d, pa + 8u * kk, bd + (uint64_t)((kk * 2048) >> 4), idesc_pv, (acc || kk > 0) ? 1u : 0u);
       };
-      // wait until the key-side bias operand of tile ti is built
-      auto bias_ready = [&](const TileInfo& ti) {
-        return ti.cls != CLS_AUG ||
-               mbar_wait(bar(B_BFULL(ti.q % NBB)), (ti.q / NBB) & 1, abort_flag, T, kHintMma);
-      };
       // query tile 1 may hold no query at all (the last CTA of a head); then only
       // tile 0's MMAs run, and they release the stages and bias operands
       const bool live1 = q0 + BM < a.Nq;
       TileInfo t0 = tiles[0];
-      bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_KFULL(0)), 0, abort_flag, T) &&
+      bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_FULL(0)), 0, abort_flag, T) &&
                 mbar_wait(bar(B_AREADY(0)), 0, abort_flag, T) &&
-                (!live1 || mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T)) && bias_ready(t0);
+                (!live1 || mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T));
       if (!ok) fail(P, abort_flag, 3);
       if (ok) {
         tc_fence_after();
@@ -505,7 +508,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_qk(1, 0, t0);
           mma_commit(bar(B_SFULL(1)));
         }
-        mma_commit(bar(B_KEMPTY(0)));
         if (t0.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(t0.q % NBB)));
         // tile 0 alone: its MMAs release every stage and bias operand
         for (int j = 0; j < nt && ok && !live1; ++j) {
@@ -513,19 +515,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int jn = j + 1, stn = jn % ST;
           const bool more = jn < nt;
           const TileInfo tn = more ? tiles[jn] : t0;
-          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma) &&
-               mbar_wait(bar(B_VFULL(st)), (j / ST) & 1, abort_flag, T, kHintMma);
+          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma);
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
           issue_pv(0, st, j > 0);
-          mma_commit(bar(B_VEMPTY(st)));
+          mma_commit(bar(B_EMPTY(st)));
           if (more) {
-            ok = mbar_wait(bar(B_KFULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma) && bias_ready(tn);
+            ok = mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma);
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
             issue_qk(0, stn, tn);
             mma_commit(bar(B_SFULL(0)));
-            mma_commit(bar(B_KEMPTY(stn)));
             if (tn.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(tn.q % NBB)));
           } else {
             mma_commit(bar(B_OFINAL(0)));
@@ -537,13 +537,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int jn = j + 1, stn = jn % ST;
           const bool more = jn < nt;
           const TileInfo tn = more ? tiles[jn] : t0;
-          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma) &&
-               mbar_wait(bar(B_VFULL(st)), (j / ST) & 1, abort_flag, T, kHintMma);
+          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma);
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
           issue_pv(0, st, j > 0);
           if (more) {
-            ok = mbar_wait(bar(B_KFULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma) && bias_ready(tn);
+            ok = mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma);
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
             issue_qk(0, stn, tn);
@@ -555,11 +554,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) { fail(P, abort_flag, 6); break; }
           tc_fence_after();
           issue_pv(1, st, j > 0);
-          mma_commit(bar(B_VEMPTY(st)));
+          mma_commit(bar(B_EMPTY(st)));
           if (more) {
             issue_qk(1, stn, tn);
             mma_commit(bar(B_SFULL(1)));
-            mma_commit(bar(B_KEMPTY(stn)));
             if (tn.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(tn.q % NBB)));
           } else {
             mma_commit(bar(B_OFINAL(1)));
