@@ -303,50 +303,6 @@ def run_graph(W, steps: int):
     return e0.elapsed_time(e1) / 1e3 / steps
 
 
-def correspond_sweep(device, iters: int = 10):
-    """Reprojection (Eq. 3-4) at a scale where it is no longer launch-bound: 4 frames of
-    180 x 320 tokens (230400 queries) against 8 retrieved chunks (32 source frames),
-    7.4 M (query, frame) pairs and 126 MB in one launch.  A sweep, not a configuration."""
-    import torch
-
-    import synth
-    from paper_2607_21848_gb300 import api
-
-    F, h, w, k = 4, 180, 320, 8
-    K = synth.pinhole(h, w, 90.0)
-    fr = synth.random_walk(synth.rng(999, "sweep"), k + 1, F, K)
-    bank = api.Bank(k + 1, F, h, w, 1, 1, 64, torch.float32, 1, device=device, with_kv=False)
-    shp = api.shape(1, 1, 64, F, h, w, torch.float32)
-    api.crc_bank_insert_poses(bank, shp, 0, synth.frame_records(fr))
-    g = torch.Generator(device=device).manual_seed(99)
-    bank.depth.copy_(torch.exp(torch.rand(bank.depth.shape, generator=g, device=device) * math.log(40.0)) * 0.5)
-    depth = bank.depth[k].clone()
-    idx = torch.arange(k, dtype=torch.int32, device=device)
-    count = torch.full((1,), k, dtype=torch.int32, device=device)
-    Nq, S = F * h * w, k * F
-    uv = torch.empty(Nq, S, 2, device=device)
-    cell = torch.empty(Nq, S, dtype=torch.int32, device=device)
-    valid = torch.empty(Nq, S, dtype=torch.uint8, device=device)
-    cur = synth.frame_records(fr[k])
-
-    def run():
-        api.crc_correspond(shp, cur, depth, bank, idx, count, k, 0.05, uv, cell, valid)
-
-    run()
-    torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(iters):
-        run()
-    e1.record()
-    torch.cuda.synchronize()
-    t = e0.elapsed_time(e1) / 1e3 / iters
-    nbytes = Nq * 4 + Nq * S * (8 + 4 + 1 + 4)
-    return {"queries": Nq, "source_frames": S, "pairs": Nq * S, "bytes": nbytes, "ms": t * 1e3,
-            "gbs": nbytes / t / 1e9, "valid_fraction": float(valid.float().mean())}
-
-
 def _bias_matrix(W):
     """lambda * B of Eq. 2 as a dense [N_q, N_k] matrix, for the materialised-bias comparator."""
     import torch
@@ -570,7 +526,11 @@ def main():
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
-    sweep = correspond_sweep(device) if not args.no_context else None
+    sweep = None
+    if not args.no_context:
+        from paper_2607_21848_gb300.sweeps import correspond_sweep
+
+        sweep = correspond_sweep(device)
 
     peaks = _peaks()
     attn_tflops = alg["flops"] / stage["attention"] / 1e12
