@@ -35,7 +35,9 @@
 // One FULL barrier per stage stands for K, V and the bias operand together, and one
 // EMPTY barrier (a commit after the tile's last PV) frees the whole stage: the
 // single MMA-issuing thread waits once per KV tile for data, since issuing a
-// 128 x 128 x 16 MMA occupies it for nearly as long as the tensor core runs it.
+// 128 x 128 x 16 MMA occupies it for nearly as long as the tensor core runs it, and
+// every wait or shared-memory load it makes costs it a round trip of issue time
+// (which tiles carry a bias/mask operand it reads from a bit mask, 32 tiles a word).
 // The query-side bias operand of each query tile is written by its own softmax
 // warpgroup whenever the source frame of the next biased tile changes.
 // TMEM (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each.  S = Q K^T is an
@@ -95,7 +97,8 @@ constexpr int OFF_V = OFF_K + ST * TILE;
 constexpr int OFF_AQ = OFF_V + ST * TILE;      // query-side bias operand, one per query tile
 constexpr int OFF_RB = OFF_AQ + NQT * AUG;     // key-side bias/mask operand ring
 constexpr int OFF_TILES = OFF_RB + NBB * AUG;
-constexpr int OFF_BAR = OFF_TILES + kMaxTiles * 12;
+constexpr int OFF_AMASK = OFF_TILES + kMaxTiles * 12;  // bit j: tile j is CLS_AUG
+constexpr int OFF_BAR = OFF_AMASK + kMaxTiles / 8;
 constexpr int NBAR = 1 + 2 * ST + 3 * NQT + 1 + NQT + 2 * NBB;
 constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
 constexpr int OFF_BOX = OFF_MISC + 64;  // per source frame: correspondence box of the CTA's queries
@@ -313,6 +316,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // KV tiles: each segment is cut into tiles of 128 keys from its start; retrieved
     // segments are cut per source frame, so that a tile has at most one frame
     const int hw = a.h * a.w;
+    uint32_t* amask = reinterpret_cast<uint32_t*>(smem + OFF_AMASK);
+    for (int i = lane; i < kMaxTiles / 32; i += 32) amask[i] = 0u;
+    __syncwarp();
     int count = 0, qa = 0;
     for (int g = 0; g < a.nseg; ++g) {
       const crc_segment sg = a.seg[g];
@@ -353,7 +359,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const unsigned m = __ballot_sync(0xffffffffu, keep);
           const unsigned ma = __ballot_sync(0xffffffffu, keep && ti.cls == CLS_AUG);
           ti.q = (uint16_t)(qa + __popc(ma & lt));
-          if (keep) tiles[count + __popc(m & lt)] = ti;
+          if (keep) {
+            const int ti_idx = count + __popc(m & lt);
+            tiles[ti_idx] = ti;
+            if (ti.cls == CLS_AUG) atomicOr(&amask[ti_idx >> 5], 1u << (ti_idx & 31));
+          }
           count += __popc(m);
           qa += __popc(ma);
         }
@@ -472,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t dv0 = sdesc_sw128(sbase + OFF_V, BOX, 1024);
       const uint64_t daq0 = sdesc_none(sbase + OFF_AQ, 128, 256);
       const uint64_t dbk0 = sdesc_none(sbase + OFF_RB, 128, 256);
-      auto issue_qk = [&](int x, int st, const TileInfo& ti) {
+      auto issue_qk = [&](int x, int st, bool aug, int bs) {
         const uint64_t ad = dq0 + (uint64_t)((x * TILE) >> 4);
         const uint64_t bd = dk0 + (uint64_t)((st * TILE) >> 4);
         const uint32_t d = tmem + TM_S + 128u * x;
@@ -481,8 +491,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t off = (uint64_t)(((kk >> 2) * BOX + (kk & 3) * 32) >> 4);
           mma_ss(d, ad + off, bd + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
-        if (ti.cls == CLS_AUG)  // + bias/mask: query-side x key-side operand, K = 16
-          mma_ss(d, daq0 + (uint64_t)((x * AUG) >> 4), dbk0 + (uint64_t)(((ti.q % NBB) * AUG) >> 4), idesc_qk, 1u);
+        if (aug)  // + bias/mask: query-side x key-side operand, K = 16
+          mma_ss(d, daq0 + (uint64_t)((x * AUG) >> 4), dbk0 + (uint64_t)((bs * AUG) >> 4), idesc_qk, 1u);
       };
       auto issue_pv = [&](int x, int st, bool acc) {
         const uint64_t bd = dv0 + (uint64_t)((st * TILE) >> 4);
@@ -495,26 +505,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       // query tile 1 may hold no query at all (the last CTA of a head); then only
       // tile 0's MMAs run, and they release the stages and bias operands
       const bool live1 = q0 + BM < a.Nq;
-      TileInfo t0 = tiles[0];
+      // Which tiles carry the bias/mask operand comes from a bit mask, one shared-memory
+      // word per 32 tiles, and their ring slots from a running count: every load this
+      // thread waits on holds up its MMA issue for a shared-memory round trip.
+      const uint32_t* amask = reinterpret_cast<const uint32_t*>(smem + OFF_AMASK);
+      uint32_t amw = amask[0];
+      const bool aug0 = (amw & 1u) != 0;
+      int bnext = aug0 ? 1 % NBB : 0;
       bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_FULL(0)), 0, abort_flag, T) &&
                 mbar_wait(bar(B_AREADY(0)), 0, abort_flag, T) &&
                 (!live1 || mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T));
       if (!ok) fail(P, abort_flag, 3);
       if (ok) {
         tc_fence_after();
-        issue_qk(0, 0, t0);
+        issue_qk(0, 0, aug0, 0);
         mma_commit(bar(B_SFULL(0)));
         if (live1) {
-          issue_qk(1, 0, t0);
+          issue_qk(1, 0, aug0, 0);
           mma_commit(bar(B_SFULL(1)));
         }
-        if (t0.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(t0.q % NBB)));
+        if (aug0) mma_commit(bar(B_BEMPTY(0)));
         // tile 0 alone: its MMAs release every stage and bias operand
         for (int j = 0; j < nt && ok && !live1; ++j) {
           const int st = j % ST;
           const int jn = j + 1, stn = jn % ST;
           const bool more = jn < nt;
-          const TileInfo tn = more ? tiles[jn] : t0;
+          if (more && (jn & 31) == 0) amw = amask[jn >> 5];
+          const bool augn = more && ((amw >> (jn & 31)) & 1u) != 0;
+          const int bs = bnext;
+          if (augn) bnext = bnext + 1 == NBB ? 0 : bnext + 1;
           ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma);
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
@@ -524,9 +543,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma);
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
-            issue_qk(0, stn, tn);
+            issue_qk(0, stn, augn, bs);
             mma_commit(bar(B_SFULL(0)));
-            if (tn.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(tn.q % NBB)));
+            if (augn) mma_commit(bar(B_BEMPTY(bs)));
           } else {
             mma_commit(bar(B_OFINAL(0)));
           }
@@ -536,7 +555,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int st = j % ST;
           const int jn = j + 1, stn = jn % ST;
           const bool more = jn < nt;
-          const TileInfo tn = more ? tiles[jn] : t0;
+          if (more && (jn & 31) == 0) amw = amask[jn >> 5];
+          const bool augn = more && ((amw >> (jn & 31)) & 1u) != 0;
+          const int bs = bnext;
+          if (augn) bnext = bnext + 1 == NBB ? 0 : bnext + 1;
           ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma);
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
@@ -545,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma);
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
-            issue_qk(0, stn, tn);
+            issue_qk(0, stn, augn, bs);
             mma_commit(bar(B_SFULL(0)));
           } else {
             mma_commit(bar(B_OFINAL(0)));
@@ -556,9 +578,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_pv(1, st, j > 0);
           mma_commit(bar(B_EMPTY(st)));
           if (more) {
-            issue_qk(1, stn, tn);
+            issue_qk(1, stn, augn, bs);
             mma_commit(bar(B_SFULL(1)));
-            if (tn.cls == CLS_AUG) mma_commit(bar(B_BEMPTY(tn.q % NBB)));
+            if (augn) mma_commit(bar(B_BEMPTY(bs)));
           } else {
             mma_commit(bar(B_OFINAL(1)));
           }
