@@ -28,16 +28,19 @@
 //   warps 4-7   softmax of query tile 1   (TMEM lanes 0-127 of S1/O1)
 //   warp  8     TMA producer: Q once, then K/V tiles of 128 keys, 2 stages each,
 //               128-byte swizzled boxes of 128 rows x 64 elements
-//   warp  9     TMEM owner and single-thread tcgen05.mma issuer
+//   warp  9     TMEM owner and tcgen05.mma issuer (the warp converged, one elected lane)
 //   warps 10-11 build, ahead of use, the key-side bias/mask operand of every tile
 //               that needs one (3-deep ring; the producer declares a stage full only
 //               once the tile's operand is built, and an MMA commit frees the slot)
 // One FULL barrier per stage stands for K, V and the bias operand together, and one
 // EMPTY barrier (a commit after the tile's last PV) frees the whole stage: the
-// single MMA-issuing thread waits once per KV tile for data, since issuing a
-// 128 x 128 x 16 MMA occupies it for nearly as long as the tensor core runs it, and
-// every wait or shared-memory load it makes costs it a round trip of issue time
-// (which tiles carry a bias/mask operand it reads from a bit mask, 32 tiles a word).
+// MMA warp waits once per KV tile for data, since issuing a 128 x 128 x 16 MMA
+// occupies it for most of the time the tensor core runs it, and every wait or
+// shared-memory load it makes costs it a round trip of issue time (which tiles
+// carry a bias/mask operand it reads from a bit mask, 32 tiles a word).  The warp
+// issues converged, one elected lane per instruction, which keeps its operands
+// uniform: 39 clocks per MMA, against 54 for a lone lane (50 against 110 while
+// the other warps of its sub-partition run arithmetic).
 // The query-side bias operand of each query tile is written by its own softmax
 // warpgroup whenever the source frame of the next biased tile changes.
 // TMEM (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each.  S = Q K^T is an
@@ -472,7 +475,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
    } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0 && nt > 0) {
+    // The whole warp runs this loop, converged, and one elected lane issues each
+    // MMA and commit; every wait's outcome is made warp-uniform before it is used.
+    if (nt > 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, 0, 0);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, HD, 0, 1);
       // descriptors of the operand bases; advancing along K adds (bytes >> 4) to the
@@ -489,10 +494,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
           const uint64_t off = (uint64_t)(((kk >> 2) * BOX + (kk & 3) * 32) >> 4);
-          mma_ss(d, ad + off, bd + off, idesc_qk, kk > 0 ? 1u : 0u);
+          mma_ss_elect(d, ad + off, bd + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
         if (aug)  // + bias/mask: query-side x key-side operand, K = 16
-          mma_ss(d, daq0 + (uint64_t)((x * AUG) >> 4), dbk0 + (uint64_t)((bs * AUG) >> 4), idesc_qk, 1u);
+          mma_ss_elect(d, daq0 + (uint64_t)((x * AUG) >> 4), dbk0 + (uint64_t)((bs * AUG) >> 4), idesc_qk, 1u);
       };
       auto issue_pv = [&](int x, int st, bool acc) {
         const uint64_t bd = dv0 + (uint64_t)((st * TILE) >> 4);
@@ -500,14 +505,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t pa = tmem + TM_S + 128u * x;
 #pragma unroll
         for (int kk = 0; kk < BN / 16; ++kk)
-          mma_ts(d, pa + 8u * kk, bd + (uint64_t)((kk * 2048) >> 4), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+          mma_ts_elect(d, pa + 8u * kk, bd + (uint64_t)((kk * 2048) >> 4), idesc_pv, (acc || kk > 0) ? 1u : 0u);
       };
       // query tile 1 may hold no query at all (the last CTA of a head); then only
       // tile 0's MMAs run, and they release the stages and bias operands
       const bool live1 = q0 + BM < a.Nq;
       // Which tiles carry the bias/mask operand comes from a bit mask, one shared-memory
-      // word per 32 tiles, and their ring slots from a running count: every load this
-      // thread waits on holds up its MMA issue for a shared-memory round trip.
+      // word per 32 tiles, and their ring slots from a running count: every load the
+      // warp waits on holds up its MMA issue for a shared-memory round trip.
       const uint32_t* amask = reinterpret_cast<const uint32_t*>(smem + OFF_AMASK);
       uint32_t amw = amask[0];
       const bool aug0 = (amw & 1u) != 0;
@@ -515,16 +520,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = mbar_wait(bar(B_QFULL()), 0, abort_flag, T) && mbar_wait(bar(B_FULL(0)), 0, abort_flag, T) &&
                 mbar_wait(bar(B_AREADY(0)), 0, abort_flag, T) &&
                 (!live1 || mbar_wait(bar(B_AREADY(1)), 0, abort_flag, T));
+      ok = __all_sync(0xffffffffu, ok);
       if (!ok) fail(P, abort_flag, 3);
       if (ok) {
         tc_fence_after();
         issue_qk(0, 0, aug0, 0);
-        mma_commit(bar(B_SFULL(0)));
+        mma_commit_elect(bar(B_SFULL(0)));
         if (live1) {
           issue_qk(1, 0, aug0, 0);
-          mma_commit(bar(B_SFULL(1)));
+          mma_commit_elect(bar(B_SFULL(1)));
         }
-        if (aug0) mma_commit(bar(B_BEMPTY(0)));
+        if (aug0) mma_commit_elect(bar(B_BEMPTY(0)));
         // tile 0 alone: its MMAs release every stage and bias operand
         for (int j = 0; j < nt && ok && !live1; ++j) {
           const int st = j % ST;
@@ -534,20 +540,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool augn = more && ((amw >> (jn & 31)) & 1u) != 0;
           const int bs = bnext;
           if (augn) bnext = bnext + 1 == NBB ? 0 : bnext + 1;
-          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma);
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma));
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
           issue_pv(0, st, j > 0);
-          mma_commit(bar(B_EMPTY(st)));
+          mma_commit_elect(bar(B_EMPTY(st)));
           if (more) {
-            ok = mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma);
+            ok = __all_sync(0xffffffffu, mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma));
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
             issue_qk(0, stn, augn, bs);
-            mma_commit(bar(B_SFULL(0)));
-            if (augn) mma_commit(bar(B_BEMPTY(bs)));
+            mma_commit_elect(bar(B_SFULL(0)));
+            if (augn) mma_commit_elect(bar(B_BEMPTY(bs)));
           } else {
-            mma_commit(bar(B_OFINAL(0)));
+            mma_commit_elect(bar(B_OFINAL(0)));
           }
         }
         // both tiles, interleaved on the tensor core
@@ -559,36 +565,36 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool augn = more && ((amw >> (jn & 31)) & 1u) != 0;
           const int bs = bnext;
           if (augn) bnext = bnext + 1 == NBB ? 0 : bnext + 1;
-          ok = mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma);
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(B_PREADY(0)), j & 1, abort_flag, T, kHintMma));
           if (!ok) { fail(P, abort_flag, 4); break; }
           tc_fence_after();
           issue_pv(0, st, j > 0);
           if (more) {
-            ok = mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma);
+            ok = __all_sync(0xffffffffu, mbar_wait(bar(B_FULL(stn)), (jn / ST) & 1, abort_flag, T, kHintMma));
             if (!ok) { fail(P, abort_flag, 5); break; }
             tc_fence_after();
             issue_qk(0, stn, augn, bs);
-            mma_commit(bar(B_SFULL(0)));
+            mma_commit_elect(bar(B_SFULL(0)));
           } else {
-            mma_commit(bar(B_OFINAL(0)));
+            mma_commit_elect(bar(B_OFINAL(0)));
           }
-          ok = mbar_wait(bar(B_PREADY(1)), j & 1, abort_flag, T, kHintMma);
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(B_PREADY(1)), j & 1, abort_flag, T, kHintMma));
           if (!ok) { fail(P, abort_flag, 6); break; }
           tc_fence_after();
           issue_pv(1, st, j > 0);
-          mma_commit(bar(B_EMPTY(st)));
+          mma_commit_elect(bar(B_EMPTY(st)));
           if (more) {
             issue_qk(1, stn, augn, bs);
-            mma_commit(bar(B_SFULL(1)));
-            if (augn) mma_commit(bar(B_BEMPTY(bs)));
+            mma_commit_elect(bar(B_SFULL(1)));
+            if (augn) mma_commit_elect(bar(B_BEMPTY(bs)));
           } else {
-            mma_commit(bar(B_OFINAL(1)));
+            mma_commit_elect(bar(B_OFINAL(1)));
           }
         }
       }
       // every MMA issued so far has retired once this barrier fires
       volatile int never = 0;
-      mma_commit(bar(B_DRAIN()));
+      mma_commit_elect(bar(B_DRAIN()));
       mbar_wait(bar(B_DRAIN()), 0, &never, 100000000ull);
     }
    }
