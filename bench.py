@@ -191,9 +191,9 @@ def run_step(W, stream, ev=None):
 LAUNCHES_PER_STEP = 4
 
 # DRAM bytes (read + write) per layer of attn_tc_kernel at the Wan-1.3B chunk shape, from one
-# ncu capture of a 2-layer launch (283.6 MB / 2); traffic grows in proportion to layers.
+# ncu capture of a 2-layer launch (283.2 MB / 2); traffic grows in proportion to layers.
 # Valid only for that shape and the kernel version it was captured on.
-ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.8e6}
+ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.6e6}
 
 
 # ---------------------------------------------------------------------------- ranks

@@ -631,7 +631,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_arrive(bar(B_AREADY(x)));
     for (int j = 0; j < nt; ++j) {
-      nxt = load_corr(a, tiles, j + 1, nt, p, row_ok, P.coef_log2);
+      // the next tile's source frame; its correspondence is fetched (a tile ahead, so
+      // that the global-load latency overlaps this tile) only when the query-side
+      // bias operand has to change for it
+      int8_t s_next = -1;
+      if (j + 1 < nt) {
+        const TileInfo tn = tiles[j + 1];
+        if (tn.cls == CLS_AUG && tn.s >= 0 && tn.s != aug_frame) s_next = tn.s;
+      }
+      if (s_next >= 0) nxt = load_corr(a, tiles, j + 1, nt, p, row_ok, P.coef_log2);
       if (ok && !mbar_wait(bar(B_SFULL(x)), j & 1, abort_flag, T, kHintSoftmax)) { fail(P, abort_flag, 7); ok = false; }
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
@@ -640,18 +648,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32u * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
       tmem_wait_ld();
-      // row max by a tree of three-input max operations
-      float mx[43];
+      // row max: eight running three-input max chains, then a final fold
+      float mx[8];
 #pragma unroll
-      for (int i = 0; i < 42; ++i)
-        mx[i] = max3f(__uint_as_float(sr[3 * i]), __uint_as_float(sr[3 * i + 1]), __uint_as_float(sr[3 * i + 2]));
-      mx[42] = fmaxf(__uint_as_float(sr[126]), __uint_as_float(sr[127]));
+      for (int i = 0; i < 8; ++i) mx[i] = fmaxf(__uint_as_float(sr[i]), __uint_as_float(sr[8 + i]));
 #pragma unroll
-      for (int i = 0; i < 14; ++i) mx[i] = max3f(mx[3 * i], mx[3 * i + 1], mx[3 * i + 2]);
-      mx[14] = mx[42];
+      for (int c = 16; c < 128; c += 16)
 #pragma unroll
-      for (int i = 0; i < 5; ++i) mx[i] = max3f(mx[3 * i], mx[3 * i + 1], mx[3 * i + 2]);
-      const float mt = max3f(max3f(mx[0], mx[1], mx[2]), mx[3], mx[4]) * sc;
+        for (int i = 0; i < 8; ++i) mx[i] = max3f(mx[i], __uint_as_float(sr[c + i]), __uint_as_float(sr[c + 8 + i]));
+      const float mt = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sc;
       // base-2 online softmax; the max is refreshed only when it grows by > 8
       const float mnew = fmaxf(m, mt);
       const bool resc = mnew > m + 8.f;
@@ -691,15 +696,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // the next tile's QK^T is issued only after this tile's P is ready, and this
       // tile's QK^T has retired: the query-side bias operand can be rewritten here
-      if (j + 1 < nt) {
-        const TileInfo tn = tiles[j + 1];
-        if (tn.cls == CLS_AUG && tn.s >= 0 && tn.s != aug_frame) {
-          uint32_t w[8];
-          aug_query_row(nxt, xc, yc, inv_sc, w);
-          store_aug_row(aq, r, w);
-          fence_async_smem();
-          aug_frame = tn.s;
-        }
+      if (s_next >= 0) {
+        uint32_t w[8];
+        aug_query_row(nxt, xc, yc, inv_sc, w);
+        store_aug_row(aq, r, w);
+        fence_async_smem();
+        aug_frame = s_next;
       }
       tmem_wait_st();
       tc_fence_before();
