@@ -373,6 +373,46 @@ def sdpa_context(W, flops: float, iters: int = 5):
 
 
 # ---------------------------------------------------------------------------- oracle arm
+def other_shapes(device, seed: int, iters: int = 5):
+    """The attention call alone on the other bf16 shapes: config 3 (k = 3, 28 080 keys, 30 layers
+    batched) and config 4 (14B-class, 40 heads, 10 800 queries, 64 800 keys, one layer).  One full
+    step first fills each cache and its correspondences through the path; then the attention is
+    timed with CUDA events.  Context for how the kernel holds beyond the headline shape."""
+    import torch
+
+    from paper_2607_21848_gb300 import api
+
+    out = {}
+    for cfg, layers in ((3, 30), (4, 1)):
+        W = setup(cfg, layers, device, seed)
+        wl = W["wl"]
+        stream = torch.cuda.current_stream()
+        run_step(W, stream)
+        flops = algorithmic(W)["flops"]
+
+        def attn():
+            api.crc_biased_attention(W["shape"], W["q"], W["cache"], W["o"], None, W["uv"], W["valid"], wl.k,
+                                     W["idx"], wl.lam, wl.sigma, 0, W["status"], stream)
+
+        for _ in range(3):
+            attn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(iters):
+            attn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / iters
+        if int(W["status"].item()) != 0:
+            raise RuntimeError(f"attention status {int(W['status'].item())} on config {cfg}")
+        out[f"config{cfg}"] = {"layers": layers, "heads": wl.H, "queries": wl.Nq, "keys": wl.n_keys, "k": wl.k,
+                               "ms": ms, "tflops": flops / ms / 1e9}
+        del W
+        torch.cuda.empty_cache()
+    return out
+
+
 def oracle_sample(cfg_id: int, layers: int, budget_s: float):
     """Time the fp64 oracle on a bounded sample of one step: the full retrieval and
     correspondence, then attention rows of one head of one layer until `budget_s`."""
@@ -526,11 +566,12 @@ def main():
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
-    sweep = None
+    sweep = shapes = None
     if not args.no_context:
         from paper_2607_21848_gb300.sweeps import correspond_sweep
 
         sweep = correspond_sweep(device)
+        shapes = other_shapes(device, rank_seed(rank))
 
     peaks = _peaks()
     attn_tflops = alg["flops"] / stage["attention"] / 1e12
@@ -565,7 +606,9 @@ def main():
     }
     if context is not None:
         line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path",
-                           "correspond_sweep": sweep}
+                           "correspond_sweep": sweep, "other_shapes": shapes}
+        for v in (shapes or {}).values():
+            v["frac_of_bf16_peak"] = v["tflops"] / peaks["bf16_sus"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cb = oracle_sample(args.config, args.layers, 10.0)
         line["cpu_baseline"] = {
