@@ -137,11 +137,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, int a_mn, in
 
 // ---- tcgen05: MMA issue and commit ------------------------------------------
 // MMA issue and commit, warp-converged: the whole warp executes them with the same
-// operands and one lane, chosen by elect.sync, issues.  Operands that are uniform across the
-// warp need no per-issue move out of the vector registers, and a converged warp
-// issues a tcgen05.mma in about 39 clocks (50 while other warps of its
-// sub-partition run arithmetic) against 54 (110) for a lone thread.  The commit
-// comes from the same elected lane, so it tracks that lane's MMAs.
+// operands and one lane, chosen by elect.sync, issues.  Measured on this GPU, a
+// converged warp issues a tcgen05.mma in about 39 clocks (50 while other warps of
+// its sub-partition run arithmetic), against 54 (110) for a lone thread under
+// `if (lane == 0)`.  The commit comes from the same elected lane, so it tracks
+// that lane's MMAs.
 __device__ __forceinline__ void mma_ss_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                              uint32_t accumulate) {
   asm volatile(
