@@ -312,6 +312,10 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
  *             an internal pipeline barrier (the output is then not valid).
  * bf16 (d = 128) runs on the tcgen05 tensor-core kernel with fp32 softmax and
  * accumulation; fp32, CRC_ATTN_SIMT or CRC_ATTN_GAUSSIAN run the SIMT kernel in fp32.
+ * The tensor-core kernel takes at most 640 KV tiles of 128 keys per call (each
+ * segment is cut into tiles from its start, a retrieved segment per frame: up to
+ * 81 920 keys) and h*w <= 65535; beyond that the call returns CRC_ERR_UNSUPPORTED
+ * before any launch, and CRC_ATTN_SIMT takes it.
  * Errors: CRC_ERR_INVALID_ARG (also unknown flag bits), CRC_ERR_SHAPE,
  * CRC_ERR_UNSUPPORTED (dtype, d, alignment, device without sm_103a), CRC_ERR_CUDA.
  */

@@ -166,6 +166,41 @@ def test_bf16_no_active_key_gives_zero_output():
     assert np.all(Og == 0) and np.all(np.isneginf(lg))
 
 
+def test_bf16_maximum_tile_count_and_one_key_beyond():
+    """640 KV tiles of 128 keys, the tensor-core kernel's limit (81 920 keys), with a biased
+    retrieved segment among them: sampled rows against the oracle.  One key more needs a
+    641st tile: the call is rejected as unsupported before any launch."""
+    F, h, w, k = 2, 8, 16, 1
+    Nc = F * h * w  # 256 queries; retrieved frames of 128 keys, one tile each
+    Nk = 640 * 128
+    g = np.random.default_rng(11)
+    segs = [(0, Nc, api.SEG_SINK, 0), (Nc, Nc, api.SEG_RETRIEVED, 0), (2 * Nc, Nk - 2 * Nc, api.SEG_WINDOW, 0)]
+    bf = lambda a: synth.bf16_round(a.astype(np.float32))  # noqa: E731
+    L, H = 1, 2
+    Q = bf(g.standard_normal((L, Nc, H, 128)))
+    Kc = bf(g.standard_normal((L, Nk + 1, H, 128)))
+    Vc = bf(g.standard_normal((L, Nk + 1, H, 128)))
+    S = k * F
+    uv = np.stack([g.uniform(-1.0, w, size=(Nc, S)), g.uniform(-1.0, h, size=(Nc, S))], -1).astype(np.float32)
+    valid = g.uniform(size=(Nc, S)) < 0.7
+    shp = api.shape(L, H, 128, F, h, w, torch.bfloat16)
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, k, 4.0, 1.0)
+    rows = np.arange(0, Nc, 9)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, (F, h, w, k), 4.0, 1.0, rows=rows)
+    _check_bf16(Og, lg, Oo, lo, rows=rows)
+    # one key more: a 641st tile
+    segs1 = segs[:2] + [(2 * Nc, Nk - 2 * Nc + 1, api.SEG_WINDOW, 0)]
+    q = _gpu.to_dev(Q, torch.bfloat16)
+    cache = api.Cache(_gpu.to_dev(Kc, torch.bfloat16), _gpu.to_dev(Vc, torch.bfloat16), segs1)
+    o = torch.full_like(q, 7.0)
+    with pytest.raises(api.CrcError) as e:
+        api.crc_biased_attention(shp, q, cache, o, None, _gpu.to_dev(uv), _gpu.to_dev(valid.astype(np.uint8)), k,
+                                 None, 4.0, 1.0)
+    torch.cuda.synchronize()
+    assert e.value.status == api._abi.CRC_ERR_UNSUPPORTED
+    assert bool((o == 7.0).all())
+
+
 def _full_size(cfg, rows, layers, heads, seed=7):
     wl = synth.make_workload(cfg)
     _, _, count, slots = _gpu.oracle_retrieve(wl)
