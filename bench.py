@@ -413,6 +413,44 @@ def other_shapes(device, seed: int, iters: int = 5):
     return out
 
 
+def opt_in_modes(W, iters: int = 3):
+    """The attention call of the headline workload in its opt-in modes, on the step's own
+    cache and correspondences: far-tile skipping and the additive-Gaussian bias on the
+    tensor-core kernel (all layers), and the Gaussian bias on the SIMT kernel (first layer
+    only: it is far slower)."""
+    import torch
+
+    from paper_2607_21848_gb300 import api
+
+    wl = W["wl"]
+    stream = torch.cuda.current_stream()
+    flops_layer = algorithmic(W)["flops"] / wl.L
+    out = {}
+    for name, flags, layers in (("skip_far", api.ATTN_SKIP_FAR, wl.L), ("gaussian", api.ATTN_GAUSSIAN, wl.L),
+                                ("gaussian_simt", api.ATTN_GAUSSIAN | api.ATTN_SIMT, 1)):
+        shp = api.shape(layers, wl.H, wl.d, wl.F, wl.h, wl.w, W["dtype"])
+        q, o = W["q"][:layers], W["o"][:layers]
+        cache = api.Cache(W["cache"].k[:layers], W["cache"].v[:layers], W["cache"].segments)
+
+        def attn():
+            api.crc_biased_attention(shp, q, cache, o, None, W["uv"], W["valid"], wl.k, W["idx"], wl.lam, wl.sigma,
+                                     flags, W["status"], stream)
+
+        attn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(iters):
+            attn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if int(W["status"].item()) != 0:
+            raise RuntimeError(f"attention status {int(W['status'].item())} in mode {name}")
+        ms = e0.elapsed_time(e1) / iters
+        out[name] = {"layers": layers, "ms": ms, "tflops": flops_layer * layers / ms / 1e9}
+    return out
+
+
 def oracle_sample(cfg_id: int, layers: int, budget_s: float):
     """Time the fp64 oracle on a bounded sample of one step: the full retrieval and
     correspondence, then attention rows of one head of one layer until `budget_s`."""
@@ -566,11 +604,12 @@ def main():
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
-    sweep = shapes = None
+    sweep = shapes = modes = None
     if not args.no_context:
         from paper_2607_21848_gb300.sweeps import correspond_sweep
 
         sweep = correspond_sweep(device)
+        modes = opt_in_modes(W)
         shapes = other_shapes(device, rank_seed(rank))
 
     peaks = _peaks()
@@ -606,7 +645,7 @@ def main():
     }
     if context is not None:
         line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path",
-                           "correspond_sweep": sweep, "other_shapes": shapes}
+                           "correspond_sweep": sweep, "other_shapes": shapes, "opt_in_modes": modes}
         for v in (shapes or {}).values():
             v["frac_of_bf16_peak"] = v["tflops"] / peaks["bf16_sus"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -283,7 +283,10 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
 #define CRC_ATTN_SIMT 1      /* force the SIMT kernel (fp32 arithmetic) for any dtype */
 #define CRC_ATTN_GAUSSIAN 2  /* opt-in: additive Gaussian bias lambda exp(-||u_k - u^||^2 / (2 sigma^2))
                                 on the biased columns instead of Eq. 2's quadratic penalty
-                                (a bonus that peaks at the correspondence; runs on the SIMT kernel) */
+                                (a bonus that peaks at the correspondence).  bf16 with d = 128 runs
+                                on the tensor-core kernel, which adds the bonus to each biased tile's
+                                scores in the softmax; otherwise the SIMT kernel.  Not combined with
+                                CRC_ATTN_SKIP_FAR, which is then ignored. */
 #define CRC_ATTN_SKIP_FAR 4  /* opt-in approximation (tensor-core kernel, Eq. 2 form): a KV tile of a
                                 retrieved frame is skipped for a block of 256 queries when every one of
                                 them has a valid correspondence in that frame and the distance from the
@@ -311,7 +314,7 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
  *   d_status  device int32 or NULL: set non-zero if a kernel gave up waiting on
  *             an internal pipeline barrier (the output is then not valid).
  * bf16 (d = 128) runs on the tcgen05 tensor-core kernel with fp32 softmax and
- * accumulation; fp32, CRC_ATTN_SIMT or CRC_ATTN_GAUSSIAN run the SIMT kernel in fp32.
+ * accumulation, in either bias form; fp32 or CRC_ATTN_SIMT run the SIMT kernel in fp32.
  * The tensor-core kernel takes at most 640 KV tiles of 128 keys per call (each
  * segment is cut into tiles from its start, a retrieved segment per frame: up to
  * 81 920 keys) and h*w <= 65535; beyond that the call returns CRC_ERR_UNSUPPORTED

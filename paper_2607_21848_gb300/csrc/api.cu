@@ -402,11 +402,14 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
   a.status = d_status;
   a.bias_form = (flags & CRC_ATTN_GAUSSIAN) ? 1 : 0;
   // skipped weights are scaled by at most 2^-64: lambda d^2 / (2 sigma^2) >= 64 ln 2
-  a.skip_far = (flags & CRC_ATTN_SKIP_FAR) && lambda > 0.f && any_ret && any_other && d_valid ? 1 : 0;
+  a.skip_far = (flags & CRC_ATTN_SKIP_FAR) && !(flags & CRC_ATTN_GAUSSIAN) && lambda > 0.f && any_ret && any_other &&
+                       d_valid
+                   ? 1
+                   : 0;
   a.skip_d2 = lambda > 0.f ? (float)(2.0 * (double)sigma * (double)sigma * 64.0 * 0.6931471805599453 / (double)lambda)
                            : INFINITY;
   cudaError_t e;
-  if (shape->dtype == CRC_BF16 && !(flags & (CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN))) {
+  if (shape->dtype == CRC_BF16 && !(flags & CRC_ATTN_SIMT)) {
     e = crc::launch_attn_tc(a, s);
     if (e == cudaErrorNotSupported) return CRC_ERR_UNSUPPORTED;
   } else {

@@ -129,6 +129,8 @@ struct TcParams {
   AttnArgs a;
   float scale_log2;  // log2(e) / sqrt(d)
   float coef_log2;   // -lambda log2(e) / (2 sigma^2)
+  float gauss_gc;    // additive-Gaussian form: lambda sqrt(d), the bonus at d = 0 in raw score units
+  float gauss_k;     // and log2(e) / (2 sigma^2), so that the bonus is gauss_gc 2^(-d^2 gauss_k)
   uint64_t timeout_ns;
 };
 
@@ -249,6 +251,9 @@ __device__ __forceinline__ void fail(const TcParams& P, volatile int* abort_flag
 
 }  // namespace
 
+// GAUSS: the opt-in additive-Gaussian bias form (CRC_ATTN_GAUSSIAN); the Eq. 2
+// instantiation carries none of its code.
+template <bool GAUSS>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ TcParams P) {
@@ -449,7 +454,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = 2 * bt + h;
         const uint32_t mask = row <= (int)ti.nact_m1 ? 0u : neg;
         uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, mask << 16};
-        if (ti.s >= 0) {
+        if (ti.s >= 0 && !GAUSS) {
           // grid cell of the key inside its source frame, relative to the frame centre
           const int loc = (int)ti.loc0 + row;
           const int yi = loc / a.w;
@@ -621,11 +626,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     // per-row correspondence of the (at most two) source frames of a tile,
     // loaded one tile ahead so that the global-load latency overlaps a tile
     Corr nxt = load_corr(a, tiles, 0, nt, p, row_ok, P.coef_log2);
-    // query-side bias/mask operand: the first tile's source frame (or no bias)
+    // query-side bias/mask operand: the first tile's source frame (or no bias).  In
+    // the additive-Gaussian form it carries only the mask multiplier, and the bonus
+    // is added to S in the softmax from the current frame's correspondence `cur`.
+    constexpr bool gauss = GAUSS;
+    const Corr none{0.f, 0.f, 0.f};
     int aug_frame = nt > 0 ? tiles[0].s : -1;
+    Corr cur = nxt;
     {
       uint32_t w[8];
-      aug_query_row(nxt, xc, yc, inv_sc, w);
+      aug_query_row(gauss ? none : nxt, xc, yc, inv_sc, w);
       store_aug_row(aq, r, w);
       fence_async_smem();
     }
@@ -648,6 +658,32 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32u * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
       tmem_wait_ld();
+      if constexpr (GAUSS) {
+        // additive-Gaussian form: S += lambda sqrt(d) 2^(-d^2 log2(e) / (2 sigma^2)) for a
+        // biased tile and a valid correspondence, with d the grid distance from the key's
+        // cell (x, y), walked column by column, to u^ of the tile's source frame
+        const TileInfo tj = tiles[j];
+        if (tj.s >= 0 && cur.cA != 0.f) {
+          const int y0 = (int)tj.loc0 / a.w;
+          float xf = (float)((int)tj.loc0 - y0 * a.w), yf = (float)y0;
+          const float wf = (float)a.w, gk = P.gauss_k, gc = P.gauss_gc;
+          float dy = cur.uyA - yf;
+          float dy2k = dy * dy * gk;
+#pragma unroll
+          for (int c = 0; c < 128; ++c) {
+            const float dx = cur.uxA - xf;
+            const float g = ex2(-fmaf(dx * dx, gk, dy2k));
+            sr[c] = __float_as_uint(fmaf(gc, g, __uint_as_float(sr[c])));
+            xf += 1.f;
+            if (xf == wf) {
+              xf = 0.f;
+              yf += 1.f;
+              dy = cur.uyA - yf;
+              dy2k = dy * dy * gk;
+            }
+          }
+        }
+      }
       // row max: eight running three-input max chains, then a final fold
       float mx[8];
 #pragma unroll
@@ -698,10 +734,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       // tile's QK^T has retired: the query-side bias operand can be rewritten here
       if (s_next >= 0) {
         uint32_t w[8];
-        aug_query_row(nxt, xc, yc, inv_sc, w);
+        aug_query_row(gauss ? none : nxt, xc, yc, inv_sc, w);
         store_aug_row(aq, r, w);
         fence_async_smem();
         aug_frame = s_next;
+        cur = nxt;
       }
       tmem_wait_st();
       tc_fence_before();
@@ -809,11 +846,14 @@ cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
   P.a = a;
   P.scale_log2 = (float)(1.4426950408889634 / sqrt((double)a.d));
   P.coef_log2 = (float)(-(double)a.lambda * 1.4426950408889634 / (2.0 * (double)a.sigma * (double)a.sigma));
+  P.gauss_gc = (float)((double)a.lambda * sqrt((double)a.d));
+  P.gauss_k = (float)(1.4426950408889634 / (2.0 * (double)a.sigma * (double)a.sigma));
   P.timeout_ns = 2000000000ull;
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  auto kernel = a.bias_form != 0 ? attn_tc_kernel<true> : attn_tc_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
   dim3 grid((a.Nq + NQT * BM - 1) / (NQT * BM), a.H, a.L);
-  attn_tc_kernel<<<grid, kThreads, SMEM_BYTES, s>>>(mq, mk, mv, P);
+  kernel<<<grid, kThreads, SMEM_BYTES, s>>>(mq, mk, mv, P);
   return cudaGetLastError();
 }
 

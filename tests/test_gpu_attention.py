@@ -262,13 +262,51 @@ def test_gaussian_form_fp32_and_bf16_match_oracle():
     assert np.abs(Og - Oo).max() <= 1e-4 and np.abs(lg - lo).max() <= 1e-4
     Oq, _ = oracle.attention(Q, Kc, Vc, uv, valid, wl.segments, wl.h, wl.w, wl.F, beta, wl.sigma, slot_chunks=slots)
     assert np.abs(Oq - Oo).max() > 1e-3  # the two bias forms differ here
-    # bf16 inputs take the SIMT kernel in this mode
+    # bf16 inputs with d = 128 take the tensor-core kernel in this mode
     shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=21, L=1)
     Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=api.ATTN_GAUSSIAN)
     Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0, bias_form="gaussian")
     Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, 2.0, 1.0, bias_form="gaussian")
     _check_bf16_peaky(Og, Oo, Oabs)
     assert np.abs(lg - lo).max() <= 1e-3
+
+
+def test_gaussian_form_tensor_core_full_size_sampled_and_against_simt():
+    """The additive-Gaussian form on the tensor-core kernel at the Wan-1.3B chunk shape
+    (three source frames, tiles cut per frame, key cells crossing grid rows): sampled rows
+    of every head against the oracle, and the whole output against the SIMT kernel."""
+    wl = synth.make_workload(2)
+    _, _, count, slots = _gpu.oracle_retrieve(wl)
+    uv, _, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
+    uv = uv.astype(np.float32)
+    uv[~valid] = 0.0
+    g = torch.Generator(device="cuda").manual_seed(17)
+    s = wl.qkv_scale
+    L = 1
+    q = (torch.randn(L, wl.Nq, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    kc = (torch.randn(L, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    vc = (torch.randn(L, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    shp = api.shape(L, wl.H, wl.d, wl.F, wl.h, wl.w, torch.bfloat16)
+    lam = 3.0
+    Og, lg = _run_attn(shp, q, kc, vc, wl.segments, uv, valid, wl.k, lam, wl.sigma, slot_chunk=slots,
+                       flags=api.ATTN_GAUSSIAN)
+    rows = np.random.default_rng(1).choice(wl.Nq, 256, replace=False)
+    rows.sort()
+    Qo, Ko, Vo = (t.float().cpu().numpy() for t in (q, kc, vc))
+    Oo, lo = oracle.attention(Qo, Ko, Vo, uv.astype(np.float64), valid, wl.segments, wl.h, wl.w, wl.F, lam,
+                              wl.sigma, slot_chunks=slots, rows=rows, bias_form="gaussian")
+    _check_bf16(Og, lg, Oo, lo, rows=rows)
+    # the bonus moves these rows by far more than the tolerance
+    Oq, _ = oracle.attention(Qo, Ko, Vo, uv.astype(np.float64), np.zeros_like(valid), wl.segments, wl.h, wl.w,
+                             wl.F, lam, wl.sigma, slot_chunks=slots, rows=rows)
+    assert np.abs(Oq - Oo).max() > 20 * 2e-2 * math.sqrt(float(np.mean(Oo ** 2)))
+    Os, ls = _run_attn(shp, q, kc, vc, wl.segments, uv, valid, wl.k, lam, wl.sigma, slot_chunk=slots,
+                       flags=api.ATTN_GAUSSIAN | api.ATTN_SIMT)
+    # two outputs each rounded to bf16 (and each within the bf16 bound of the exact result):
+    # their difference is bounded by twice the single-path tolerance
+    err, rel, _ = _gpu.attn_errors(Og, Os.astype(np.float64))
+    assert err <= 2e-2 and rel <= 4e-2, (err, rel)
+    assert np.abs(lg - ls).max() <= 1e-3
 
 
 def test_unknown_attention_flags_are_rejected():
