@@ -191,9 +191,9 @@ def run_step(W, stream, ev=None):
 LAUNCHES_PER_STEP = 4
 
 # DRAM bytes (read + write) per layer of attn_tc_kernel at the Wan-1.3B chunk shape, from one
-# ncu capture of a 2-layer launch (283.2 MB / 2); traffic grows in proportion to layers.
+# ncu capture of a 2-layer launch (283.8 MB / 2); traffic grows in proportion to layers.
 # Valid only for that shape and the kernel version it was captured on.
-ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.6e6}
+ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.9e6}
 
 
 # ---------------------------------------------------------------------------- ranks
@@ -275,6 +275,30 @@ def run_e2e(W, stream, steps: int):
     h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + W["frames"].nbytes
     d2h = host_out[0].numel() * host_out[0].element_size()
     return e0.elapsed_time(e1) / 1e3 / steps, h2d, d2h
+
+
+def link_gbs(W, reps: int = 3):
+    """Pinned host <-> device copy bandwidth, measured on the step's largest input (Q):
+    the end-to-end figure cannot beat the step's copy bytes over these rates."""
+    import torch
+
+    src = W["q"]
+    host = torch.empty(src.shape, dtype=src.dtype, pin_memory=True)
+    dev = torch.empty_like(src)
+    nbytes = src.numel() * src.element_size()
+    out = {}
+    for name, fn in (("h2d", lambda: dev.copy_(host, non_blocking=True)),
+                     ("d2h", lambda: host.copy_(src, non_blocking=True))):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        out[name] = nbytes * reps / (e0.elapsed_time(e1) / 1e3) / 1e9
+    return out
 
 
 # ---------------------------------------------------------------------------- context
@@ -601,6 +625,7 @@ def main():
 
     barrier()
     e2e_s, h2d, d2h = run_e2e(W, stream, max(3, min(args.steps, 20)))
+    link = link_gbs(W)
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
@@ -637,7 +662,9 @@ def main():
                      "traffic_algorithmic": alg["attn_bytes"]},
         "e2e": {"value": whole_job_tflops(alg["flops"], e2e_s, world), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
-                "pipelining": "two device buffer sets; uploads and downloads on two copy streams overlap the kernels"},
+                "pipelining": "two device buffer sets; uploads and downloads on two copy streams overlap the kernels",
+                "link_gbs": link,
+                "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6},
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
                   "note": "one step captured in a CUDA graph and replayed"},
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,
