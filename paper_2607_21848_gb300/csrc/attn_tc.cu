@@ -38,9 +38,9 @@
 // occupies it for most of the time the tensor core runs it, and every wait or
 // shared-memory load it makes costs it a round trip of issue time (which tiles
 // carry a bias/mask operand it reads from a bit mask, 32 tiles a word).  The warp
-// issues converged, one elected lane per instruction, which keeps its operands
-// uniform: 39 clocks per MMA, against 54 for a lone lane (50 against 110 while
-// the other warps of its sub-partition run arithmetic).
+// issues converged, one elected lane per instruction: measured, 39 clocks per MMA
+// against 54 for a lone lane (50 against 110 while the other warps of its
+// sub-partition run arithmetic).
 // The query-side bias operand of each query tile is written by its own softmax
 // warpgroup whenever the source frame of the next biased tile changes.
 // TMEM (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each.  S = Q K^T is an
@@ -53,6 +53,11 @@
 // than 2^8 (exact: the same max normalises P, O and the row sum); O in TMEM is
 // rescaled only on those rare steps.  Keys outside every segment and retrieved
 // slots without a chunk produce no tile at all.
+//
+// The opt-in additive-Gaussian form (lambda exp(-d^2 / (2 sigma^2)) on the same
+// columns) has no low-rank expansion.  Its instantiation (GAUSS = true) keeps only
+// the mask in the K = 16 operand and adds the bonus to S in the softmax, column by
+// column, before the row max.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
