@@ -233,6 +233,12 @@ def test_bf16_config2_full_size_sampled_rows():
     _full_size(2, rows, [0], range(12))
 
 
+def test_bf16_config2_one_layer_every_row_and_head():
+    """The full comparison at the Wan-1.3B chunk shape: every query row of every head of
+    one layer against the fp64 oracle (all 18 720 keys)."""
+    _full_size(2, None, [0], range(12))
+
+
 def test_bf16_config3_30_layers_sampled():
     # 512 sampled query rows, all 12 heads, first, middle and last of the 30 layers
     rows = np.random.default_rng(1).choice(4680, 512, replace=False)
