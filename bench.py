@@ -475,6 +475,28 @@ def opt_in_modes(W, iters: int = 3):
     return out
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    import platform
+    import subprocess
+
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
+
+
 def oracle_sample(cfg_id: int, layers: int, budget_s: float):
     """Time the fp64 oracle on a bounded sample of one step: the full retrieval and
     correspondence, then attention rows of one head of one layer until `budget_s`."""
@@ -548,7 +570,7 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": _config(wl, args),
-            "cpu_baseline": {"value": tfl, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle",
+            "cpu_baseline": {"value": tfl, "unit": "TFLOP/s", "cores": os.cpu_count(), "cpu": cpu_model(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": tfl, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -683,7 +705,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cb = oracle_sample(args.config, args.layers, 10.0)
         line["cpu_baseline"] = {
-            "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["threads"], "kind": "oracle",
+            "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["threads"], "cpu": cpu_model(), "kind": "oracle",
             "sample": f"fp64 oracle: full retrieval + correspondence ({cb['t_front']:.2f} s), then {cb['rows']} of "
                       f"{wl.Nq} attention rows of one head of one layer against all {wl.n_keys} keys "
                       f"({cb['t_attn']:.1f} s); TFLOP/s = sampled attention FLOP / sampled time; a full step "
