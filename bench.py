@@ -475,6 +475,57 @@ def opt_in_modes(W, iters: int = 3):
     return out
 
 
+def stream_context(device, seed: int):
+    """The long-horizon loop-closure stream (config 5: Wan-1.3B head shape, 30 layers,
+    k = 2, 200 chunk steps on a closed camera loop) through ChunkStream, eager, with no
+    host synchronisation between steps.  Depths and frame records are staged before the
+    timed loop; each step's retrieved-slot indices are copied on the device so that the
+    active keys, and from them the algorithmic FLOP, are counted afterwards."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2607_21848_gb300 import stream as crs
+
+    wl = synth.make_workload(5)
+    cfg = crs.StreamConfig(L=wl.L, H=wl.H, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2,
+                           capacity=wl.bank_size, num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c,
+                           cos_tau_v=wl.cos_tau_v, delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps)
+    st = crs.ChunkStream(cfg, device=device)
+    Nc = cfg.Nc
+    g = torch.Generator(device=device).manual_seed(seed)
+    sc = wl.qkv_scale
+    kv = [((torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device=device) * sc).bfloat16(),
+           (torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device=device) * sc).bfloat16()) for _ in range(3)]
+    q = (torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device=device) * sc).bfloat16()
+    o = torch.empty_like(q)
+    steps = wl.bank_size
+    depth = torch.from_numpy(np.stack([wl.depth_of(n) for n in range(steps)])).to(device)
+    recs = [synth.frame_records(wl.bank_frames[n]) for n in range(steps)]
+    idx_hist = torch.empty(steps, cfg.k, dtype=torch.int32, device=device)
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for n in range(steps):
+        kn, vn = kv[n % 3]
+        st.step(n, recs[n], depth[n], kn, vn, q, o, stream=stream)
+        idx_hist[n].copy_(st.idx, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if int(st.status.item()) != 0:
+        raise RuntimeError(f"stream: attention status {int(st.status.item())}")
+    total_s = e0.elapsed_time(e1) / 1e3
+    idx = idx_hist.cpu().numpy()
+    flops = 0.0
+    for n in range(steps):
+        keys = sum(length for _, length, _, _ in st.segments(n)) - Nc * int((idx[n] < 0).sum())
+        flops += 4.0 * Nc * keys * cfg.d * cfg.H * cfg.L
+    return {"steps": steps, "layers": cfg.L, "k": cfg.k, "ms_per_step": total_s / steps * 1e3,
+            "tflops": flops / total_s / 1e12, "steps_with_retrieval": int((idx >= 0).any(axis=1).sum()),
+            "note": "whole stream step (update, retrieve, correspond, attention), eager, no host sync"}
+
+
 def cpu_model() -> str:
     """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
     import platform
@@ -654,12 +705,13 @@ def main():
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
-    sweep = shapes = modes = None
+    sweep = shapes = modes = stream_ctx = None
     if not args.no_context:
         from paper_2607_21848_gb300.sweeps import correspond_sweep
 
         sweep = correspond_sweep(device)
         modes = opt_in_modes(W)
+        stream_ctx = stream_context(device, rank_seed(rank))
         shapes = other_shapes(device, rank_seed(rank))
 
     peaks = _peaks()
@@ -699,7 +751,8 @@ def main():
     }
     if context is not None:
         line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path",
-                           "correspond_sweep": sweep, "other_shapes": shapes, "opt_in_modes": modes}
+                           "correspond_sweep": sweep, "other_shapes": shapes, "opt_in_modes": modes,
+                           "stream": stream_ctx}
         for v in (shapes or {}).values():
             v["frac_of_bf16_peak"] = v["tflops"] / peaks["bf16_sus"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
