@@ -223,21 +223,26 @@ def whole_job_tflops(flops_per_rank_step: float, step_s: float, world: int) -> f
 E2E_INPUTS = ("q", "k_new", "v_new", "depth")
 
 
+E2E_BUFFERS = 3
+
+
 def run_e2e(W, stream, steps: int):
     """The step through the public API with host buffers, pipelined on two copy streams.
 
     Every step copies its inputs (Q, the new chunk's K/V, its depth) from pinned host
-    memory and copies O back.  Two device buffer sets let step i+1's upload and step
-    i-1's download overlap step i's kernels.  Returns (seconds per step, h2d, d2h bytes)."""
+    memory and copies O back.  NB device buffer sets let the uploads run up to NB - 1
+    steps ahead and the downloads trail, both overlapping the kernels, so that jitter of
+    the host link is absorbed.  Returns (seconds per step, h2d, d2h bytes)."""
     import torch
 
+    NB = E2E_BUFFERS
     host_in = {k: W[k].cpu().pin_memory() for k in E2E_INPUTS}
-    dev = [W, dict(W, **{k: torch.empty_like(W[k]) for k in E2E_INPUTS + ("o",)})]
-    host_out = [torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True) for _ in range(2)]
+    dev = [W] + [dict(W, **{k: torch.empty_like(W[k]) for k in E2E_INPUTS + ("o",)}) for _ in range(NB - 1)]
+    host_out = [torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True) for _ in range(NB)]
     h2d_s, d2h_s = torch.cuda.Stream(), torch.cuda.Stream()
-    in_ready = [torch.cuda.Event() for _ in range(2)]
-    done = [torch.cuda.Event() for _ in range(2)]
-    out_read = [torch.cuda.Event() for _ in range(2)]
+    in_ready = [torch.cuda.Event() for _ in range(NB)]
+    done = [torch.cuda.Event() for _ in range(NB)]
+    out_read = [torch.cuda.Event() for _ in range(NB)]
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
@@ -246,22 +251,23 @@ def run_e2e(W, stream, steps: int):
     d2h_s.wait_stream(stream)
 
     def upload(i):
-        b = i % 2
+        b = i % NB
         with torch.cuda.stream(h2d_s):
-            if i >= 2:
-                h2d_s.wait_event(done[b])  # step i-2 has finished reading buffer b
+            if i >= NB:
+                h2d_s.wait_event(done[b])  # step i-NB has finished reading buffer b
             for k in E2E_INPUTS:
                 dev[b][k].copy_(host_in[k], non_blocking=True)
             in_ready[b].record(h2d_s)
 
-    upload(0)
+    for i in range(min(NB - 1, steps)):
+        upload(i)
     for i in range(steps):
-        b = i % 2
-        if i + 1 < steps:
-            upload(i + 1)
+        b = i % NB
+        if i + NB - 1 < steps:
+            upload(i + NB - 1)
         stream.wait_event(in_ready[b])
-        if i >= 2:
-            stream.wait_event(out_read[b])  # O of step i-2 has left buffer b
+        if i >= NB:
+            stream.wait_event(out_read[b])  # O of step i-NB has left buffer b
         run_step(dev[b], stream)
         done[b].record(stream)
         with torch.cuda.stream(d2h_s):
@@ -741,7 +747,8 @@ def main():
                      "traffic_algorithmic": alg["attn_bytes"]},
         "e2e": {"value": whole_job_tflops(alg["flops"], e2e_s, world), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
-                "pipelining": "two device buffer sets; uploads and downloads on two copy streams overlap the kernels",
+                "pipelining": f"{E2E_BUFFERS} device buffer sets; uploads run up to {E2E_BUFFERS - 1} steps ahead "
+                              "and downloads trail on two copy streams, overlapping the kernels",
                 "link_gbs": link,
                 "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6},
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
