@@ -230,16 +230,19 @@ def run_e2e(W, stream, steps: int):
     """The step through the public API with host buffers, pipelined on two copy streams.
 
     Every step copies its inputs (Q, the new chunk's K/V, its depth) from pinned host
-    memory and copies O back.  NB device buffer sets let the uploads run up to NB - 1
-    steps ahead and the downloads trail, both overlapping the kernels, so that jitter of
-    the host link is absorbed.  Returns (seconds per step, h2d, d2h bytes)."""
+    memory and copies O back, on one copy stream: the step's copies fit in its kernel
+    time one direction at a time, and running both directions at once made the host
+    side slow and erratic.  NB device buffer sets let the uploads run up to NB - 1 steps
+    ahead and the downloads trail, overlapping the kernels.  Returns (seconds per step,
+    h2d, d2h bytes)."""
     import torch
 
     NB = E2E_BUFFERS
     host_in = {k: W[k].cpu().pin_memory() for k in E2E_INPUTS}
     dev = [W] + [dict(W, **{k: torch.empty_like(W[k]) for k in E2E_INPUTS + ("o",)}) for _ in range(NB - 1)]
     host_out = [torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True) for _ in range(NB)]
-    h2d_s, d2h_s = torch.cuda.Stream(), torch.cuda.Stream()
+    h2d_s = torch.cuda.Stream()
+    d2h_s = h2d_s  # one copy stream for both directions
     in_ready = [torch.cuda.Event() for _ in range(NB)]
     done = [torch.cuda.Event() for _ in range(NB)]
     out_read = [torch.cuda.Event() for _ in range(NB)]
@@ -747,8 +750,8 @@ def main():
                      "traffic_algorithmic": alg["attn_bytes"]},
         "e2e": {"value": whole_job_tflops(alg["flops"], e2e_s, world), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
-                "pipelining": f"{E2E_BUFFERS} device buffer sets; uploads run up to {E2E_BUFFERS - 1} steps ahead "
-                              "and downloads trail on two copy streams, overlapping the kernels",
+                "pipelining": f"{E2E_BUFFERS} device buffer sets; on one copy stream, uploads run up to "
+                              f"{E2E_BUFFERS - 1} steps ahead and downloads trail, overlapping the kernels",
                 "link_gbs": link,
                 "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6},
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
