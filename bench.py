@@ -80,7 +80,7 @@ class ClockSampler:
     def summary(self):
         if self.proc is None or not self.path:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in open(self.path):
             parts = [x.strip() for x in line.split(",")]
@@ -91,12 +91,16 @@ class ClockSampler:
                 mx.append(float(parts[1]))
             except ValueError:
                 continue
+            try:
+                pw.append(float(parts[2]))
+            except ValueError:
+                pass
             for nm, val in zip(names, parts[4:8]):
                 if val.lower().startswith("active"):
                     reasons.add(nm)
         os.unlink(self.path)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "samples": len(sm), "reasons": sorted(reasons)}
+                "power_w": statistics.median(pw) if pw else None, "samples": len(sm), "reasons": sorted(reasons)}
 
 
 # ---------------------------------------------------------------------------- workload
@@ -709,7 +713,8 @@ def main():
     value = whole_job_tflops(alg["flops"], step_s, world)
 
     barrier()
-    e2e_s, h2d, d2h = run_e2e(W, stream, max(3, args.steps))  # as many steps as the device timing
+    with ClockSampler(local) as clk_e2e:
+        e2e_s, h2d, d2h = run_e2e(W, stream, max(3, args.steps))  # as many steps as the device timing
     link = link_gbs(W)
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
@@ -753,6 +758,7 @@ def main():
                 "pipelining": f"{E2E_BUFFERS} device buffer sets; on one copy stream, uploads run up to "
                               f"{E2E_BUFFERS - 1} steps ahead and downloads trail, overlapping the kernels",
                 "link_gbs": link,
+                "clocks": clk_e2e.summary(),
                 "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6},
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
                   "note": "one step captured in a CUDA graph and replayed"},
