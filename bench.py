@@ -12,7 +12,12 @@ call.  Inputs are resident in HBM and far larger than L2 (K/V cache 3.4 GB).
 
 Prints one JSON line.  `value` is the biased-attention algorithmic TFLOP/s of
 the whole step (4 N_q N_k d H L per step / step time, summed over ranks);
-per-stage GB/s for retrieval and reprojection ride along in `stages`.
+per-stage GB/s for retrieval and reprojection ride along in `stages`, the
+attention kernel's roofline in `roofline`, the same step through host buffers in
+`e2e`, and, unless --no-context, measurements beside the headline in `context`
+(PyTorch SDPA on the same tensors, a reprojection sweep, the opt-in attention
+modes, the 200-step loop-closure stream, and the attention on the k = 3 and
+14B-class shapes).
 """
 
 from __future__ import annotations
@@ -658,7 +663,9 @@ def main():
     ap.add_argument("--layers", type=int, default=30)
     ap.add_argument("--impl", default="crc", choices=["crc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-context", action="store_true", help="skip the PyTorch SDPA comparators")
+    ap.add_argument("--no-context", action="store_true",
+                    help="skip the context block: PyTorch SDPA comparators, the reprojection sweep, the opt-in "
+                         "attention modes, the loop-closure stream and the other shapes")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
