@@ -416,16 +416,18 @@ def sdpa_context(W, flops: float, iters: int = 5):
 
 # ---------------------------------------------------------------------------- oracle arm
 def other_shapes(device, seed: int, iters: int = 5):
-    """The attention call alone on the other bf16 shapes: config 3 (k = 3, 28 080 keys, 30 layers
-    batched) and config 4 (14B-class, 40 heads, 10 800 queries, 64 800 keys, one layer).  One full
-    step first fills each cache and its correspondences through the path; then the attention is
-    timed with CUDA events.  Context for how the kernel holds beyond the headline shape."""
+    """The attention call alone on the other bf16 shapes: Wan-1.3B with k = 3 (28 080 keys, 30
+    layers batched) and the 14B-class 720p shape (40 heads, 10 800 queries, 64 800 keys, one
+    layer).  One full step first fills each cache and its correspondences through the path;
+    then the attention is timed with CUDA events.  Context for how the kernel holds beyond the
+    headline shape."""
     import torch
 
+    import synth
     from paper_2607_21848_gb300 import api
 
     out = {}
-    for cfg, layers in ((3, 30), (4, 1)):
+    for cfg, layers in ((3, 30), (4, 1)):  # synth workloads: Wan-1.3B k = 3, and 14B-class 720p
         W = setup(cfg, layers, device, seed)
         wl = W["wl"]
         stream = torch.cuda.current_stream()
@@ -448,7 +450,7 @@ def other_shapes(device, seed: int, iters: int = 5):
         ms = e0.elapsed_time(e1) / iters
         if int(W["status"].item()) != 0:
             raise RuntimeError(f"attention status {int(W['status'].item())} on config {cfg}")
-        out[f"config{cfg}"] = {"layers": layers, "heads": wl.H, "queries": wl.Nq, "keys": wl.n_keys, "k": wl.k,
+        out[synth.WORKLOAD_NAMES[cfg]] = {"layers": layers, "heads": wl.H, "queries": wl.Nq, "keys": wl.n_keys, "k": wl.k,
                                "ms": ms, "tflops": flops / ms / 1e9}
         del W
         torch.cuda.empty_cache()
@@ -494,7 +496,7 @@ def opt_in_modes(W, iters: int = 3):
 
 
 def stream_context(device, seed: int):
-    """The long-horizon loop-closure stream (config 5: Wan-1.3B head shape, 30 layers,
+    """The long-horizon loop-closure stream (Wan-1.3B head shape, 30 layers,
     k = 2, 200 chunk steps on a closed camera loop) through ChunkStream, eager, with no
     host synchronisation between steps.  Depths and frame records are staged before the
     timed loop; each step's retrieved-slot indices are copied on the device so that the

@@ -346,11 +346,21 @@ def _segments(Nc: int, k: int, window_chunks: int) -> Tuple[List[Tuple[int, int,
     return segs, off
 
 
+# The five workloads, by what they are (the index selects one in make_workload).
+WORKLOAD_NAMES = {
+    1: "tiny_fp32_8x8_k1",           # 1 head, d = 64, 2 frames of 8x8, 512 keys, fp32
+    2: "wan1.3b_30x52_k1",           # 12 heads, d = 128, 3 frames of 30x52, 18 720 keys, bank 64
+    3: "wan1.3b_30x52_k3_bank2000",  # as above with k = 3, 28 080 keys, 30 layers per call
+    4: "14b_720p_45x80_k2",          # 40 heads, 3 frames of 45x80, 64 800 keys, bank 500
+    5: "wan1.3b_loop_stream_k2",     # the 200-step loop-closure stream, 30 layers
+}
+
+
 def make_workload(cfg: int, *, layers: Optional[int] = None, heads: Optional[int] = None,
                   bank: Optional[int] = None, grid: Optional[Tuple[int, int]] = None,
                   seed: Optional[int] = None) -> Workload:
-    """Build config `cfg` (1..5).  `layers`, `heads`, `bank` and `grid` shrink it for
-    seconds-scale parity runs while keeping its structure."""
+    """Build workload `cfg` of WORKLOAD_NAMES (1..5).  `layers`, `heads`, `bank` and `grid`
+    shrink it for seconds-scale parity runs while keeping its structure."""
     seed = 1000 + cfg if seed is None else seed
     gp = rng(seed, "poses")
     if cfg == 1:

@@ -89,7 +89,7 @@ def _check_bf16_peaky(Og, Oo, Oabs):
     assert worst <= 1.0, worst
 
 
-def test_fp32_config1_matches_oracle_1e4():
+def test_fp32_tiny_8x8_matches_oracle_1e4():
     wl = synth.make_workload(1)
     idx, _, count, slots = _gpu.oracle_retrieve(wl)
     uv, cell, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
@@ -227,26 +227,26 @@ def _full_size(cfg, rows, layers, heads, seed=7):
     assert valid.mean() > 0.05
 
 
-def test_bf16_config2_full_size_sampled_rows():
+def test_bf16_wan13b_chunk_full_size_sampled_rows():
     rows = np.random.default_rng(0).choice(4680, 1024, replace=False)
     rows.sort()
     _full_size(2, rows, [0], range(12))
 
 
-def test_bf16_config2_one_layer_every_row_and_head():
+def test_bf16_wan13b_chunk_one_layer_every_row_and_head():
     """The full comparison at the Wan-1.3B chunk shape: every query row of every head of
     one layer against the fp64 oracle (all 18 720 keys)."""
     _full_size(2, None, [0], range(12))
 
 
-def test_bf16_config3_30_layers_sampled():
+def test_bf16_wan13b_k3_30_layers_sampled():
     # 512 sampled query rows, all 12 heads, first, middle and last of the 30 layers
     rows = np.random.default_rng(1).choice(4680, 512, replace=False)
     rows.sort()
     _full_size(3, rows, [0, 17, 29], range(12))
 
 
-def test_bf16_config4_full_size_sampled():
+def test_bf16_14b_720p_full_size_sampled():
     # 14B / 720p shape: 512 sampled query rows of all 40 heads against all 64800 keys
     rows = np.random.default_rng(2).choice(10800, 512, replace=False)
     rows.sort()
