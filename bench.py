@@ -423,7 +423,6 @@ def other_shapes(device, seed: int, iters: int = 5):
     headline shape."""
     import torch
 
-    import synth
     from paper_2607_21848_gb300 import api
 
     out = {}
@@ -450,7 +449,7 @@ def other_shapes(device, seed: int, iters: int = 5):
         ms = e0.elapsed_time(e1) / iters
         if int(W["status"].item()) != 0:
             raise RuntimeError(f"attention status {int(W['status'].item())} on config {cfg}")
-        out[synth.WORKLOAD_NAMES[cfg]] = {"layers": layers, "heads": wl.H, "queries": wl.Nq, "keys": wl.n_keys, "k": wl.k,
+        out[wl.name] = {"layers": layers, "heads": wl.H, "queries": wl.Nq, "keys": wl.n_keys, "k": wl.k,
                                "ms": ms, "tflops": flops / ms / 1e9}
         del W
         torch.cuda.empty_cache()

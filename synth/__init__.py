@@ -23,7 +23,7 @@ from .workloads import (  # noqa: F401
     make_kv_pool,
     bf16_round,
     frame_records,
-    CONFIG_NAMES,
+    WORKLOAD_NAMES,
     rng,
     random_walk,
     circle_loop,

@@ -35,12 +35,13 @@ SEG_SINK = 0
 SEG_RETRIEVED = 1
 SEG_WINDOW = 2
 
-CONFIG_NAMES = {
-    1: "tiny_fp32_8x8_k1",
-    2: "wan1.3b_30x52_k1",
-    3: "wan1.3b_30x52_k3_30L",
-    4: "14b_45x80_k2",
-    5: "wan1.3b_loop_stream_k2",
+# The five workloads, by what they are (make_workload takes the index).
+WORKLOAD_NAMES = {
+    1: "tiny_fp32_8x8_k1",        # 1 head, d = 64, 2 frames of 8x8, 512 keys, fp32
+    2: "wan1.3b_30x52_k1",        # 12 heads, d = 128, 3 frames of 30x52, 18 720 keys, bank 64
+    3: "wan1.3b_30x52_k3_30L",    # as above with k = 3, 28 080 keys, bank 2000, 30 layers per call
+    4: "14b_45x80_k2",            # 40 heads, 3 frames of 45x80, 64 800 keys, bank 500
+    5: "wan1.3b_loop_stream_k2",  # the 200-step loop-closure stream, 30 layers
 }
 
 _PURPOSES = ("poses", "depth", "q", "k", "v", "bank", "scene", "pool", "step", "sweep")
@@ -346,16 +347,6 @@ def _segments(Nc: int, k: int, window_chunks: int) -> Tuple[List[Tuple[int, int,
     return segs, off
 
 
-# The five workloads, by what they are (the index selects one in make_workload).
-WORKLOAD_NAMES = {
-    1: "tiny_fp32_8x8_k1",           # 1 head, d = 64, 2 frames of 8x8, 512 keys, fp32
-    2: "wan1.3b_30x52_k1",           # 12 heads, d = 128, 3 frames of 30x52, 18 720 keys, bank 64
-    3: "wan1.3b_30x52_k3_bank2000",  # as above with k = 3, 28 080 keys, 30 layers per call
-    4: "14b_720p_45x80_k2",          # 40 heads, 3 frames of 45x80, 64 800 keys, bank 500
-    5: "wan1.3b_loop_stream_k2",     # the 200-step loop-closure stream, 30 layers
-}
-
-
 def make_workload(cfg: int, *, layers: Optional[int] = None, heads: Optional[int] = None,
                   bank: Optional[int] = None, grid: Optional[Tuple[int, int]] = None,
                   seed: Optional[int] = None) -> Workload:
@@ -426,7 +417,7 @@ def make_workload(cfg: int, *, layers: Optional[int] = None, heads: Optional[int
         E, w_v, tau_c, cos_tau_v, delta, eps = 20.0, 0.5, 0.1, math.cos(math.radians(45.0)), 3, 0.05
         scale = 1.0 / math.sqrt(128.0)
     num_slabs = min(B, 16)
-    return Workload(cfg=cfg, name=CONFIG_NAMES[cfg], H=H, d=d, F=F, h=h, w=w, L=L, k=k, dtype=dtype,
+    return Workload(cfg=cfg, name=WORKLOAD_NAMES[cfg], H=H, d=d, F=F, h=h, w=w, L=L, k=k, dtype=dtype,
                     segments=segs, n_keys=Nk, E=E, w_v=w_v, tau_c=tau_c, cos_tau_v=cos_tau_v,
                     delta=delta, lam=2.0, sigma=1.0, eps=eps, bank_frames=walk, cur_frames=cur,
                     n=B if cfg != 5 else B - 1, num_slabs=num_slabs, seed=seed, dmin=dmin, dmax=dmax,
