@@ -17,101 +17,108 @@ import pytest
 
 import oracle
 
-hyp = pytest.importorskip("hypothesis")
-st = pytest.importorskip("hypothesis.strategies")
-given, settings = hyp.given, hyp.settings
+try:
+    import hypothesis as hyp
+    import hypothesis.strategies as st
+except ImportError:  # the tests below need hypothesis; without it one placeholder skips
+    hyp = None
 
-SETTINGS = dict(max_examples=25, deadline=None)
-
-
-def _rotation(g):
-    """A uniformly random rotation (QR of a Gaussian matrix, sign-fixed, det +1)."""
-    qm, rm = np.linalg.qr(g.normal(size=(3, 3)))
-    qm = qm * np.sign(np.diag(rm))
-    if np.linalg.det(qm) < 0:
-        qm[:, 0] = -qm[:, 0]
-    return qm
+if hyp is None:
+    def test_property_pins_need_hypothesis():
+        pytest.skip("hypothesis is not installed")
+else:
+    given, settings = hyp.given, hyp.settings
+    SETTINGS = dict(max_examples=25, deadline=None)
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 2**31 - 1), B=st.integers(1, 40), k=st.integers(1, 6),
-       w_v=st.floats(0.0, 1.0), tau_c=st.floats(0.2, 4.0), cos_tau_v=st.floats(-1.0, 0.9))
-def test_retrieval_invariant_under_one_rigid_motion(seed, B, k, w_v, tau_c, cos_tau_v):
-    g = np.random.default_rng(seed)
-    bc = g.normal(size=(B, 3)) * 3.0
-    bv = g.normal(size=(B, 3))
-    bv /= np.linalg.norm(bv, axis=1, keepdims=True)
-    cn = g.normal(size=3)
-    vn = g.normal(size=3)
-    vn /= np.linalg.norm(vn)
-    E, n, delta = 2.0, B + 2, 2
-    idx, score, count = oracle.retrieve(bc, bv, cn, vn, n, E, w_v, tau_c, cos_tau_v, delta, k)
-    R, t = _rotation(g), g.normal(size=3) * 10.0
-    idx2, score2, count2 = oracle.retrieve(bc @ R.T + t, bv @ R.T, R @ cn + t, R @ vn, n, E, w_v, tau_c, cos_tau_v,
-                                           delta, k)
-    # the motion changes scores and gate terms only by rounding; skip draws that sit on a
-    # gate threshold or have two candidates within rounding of each other
-    s, dist, dot = oracle.crc_oracle.retrieval_terms(bc, bv, cn, vn, E, w_v)
-    hyp.assume(np.all(np.abs(dist - tau_c) > 1e-9) and np.all(np.abs(dot - cos_tau_v) > 1e-9))
-    ss = np.sort(s)
-    hyp.assume(B < 2 or np.min(np.diff(ss)) > 1e-9)
-    assert count2 == count
-    assert list(idx2) == list(idx)
-    np.testing.assert_allclose(score2[:count], score[:count], rtol=1e-12, atol=1e-12)
+    def _rotation(g):
+        """A uniformly random rotation (QR of a Gaussian matrix, sign-fixed, det +1)."""
+        qm, rm = np.linalg.qr(g.normal(size=(3, 3)))
+        qm = qm * np.sign(np.diag(rm))
+        if np.linalg.det(qm) < 0:
+            qm[:, 0] = -qm[:, 0]
+        return qm
 
 
-def _attn_case(g, h, w, F, d):
-    Nc = F * h * w
-    segs = [(0, Nc, oracle.crc_oracle.SEG_SINK, 0), (Nc, Nc, oracle.crc_oracle.SEG_RETRIEVED, 0),
-            (2 * Nc, Nc, oracle.crc_oracle.SEG_WINDOW, 0)]
-    Nk = 3 * Nc
-    Q = g.normal(size=(1, Nc, 1, d))
-    Kc = g.normal(size=(1, Nk, 1, d))
-    Vc = g.normal(size=(1, Nk, 1, d))
-    uv = g.uniform(-0.5, max(h, w), size=(Nc, F, 2))
-    valid = g.uniform(size=(Nc, F)) < 0.7
-    return Q, Kc, Vc, uv, valid, segs
+    @settings(**SETTINGS)
+    @given(seed=st.integers(0, 2**31 - 1), B=st.integers(1, 40), k=st.integers(1, 6),
+           w_v=st.floats(0.0, 1.0), tau_c=st.floats(0.2, 4.0), cos_tau_v=st.floats(-1.0, 0.9))
+    def test_retrieval_invariant_under_one_rigid_motion(seed, B, k, w_v, tau_c, cos_tau_v):
+        g = np.random.default_rng(seed)
+        bc = g.normal(size=(B, 3)) * 3.0
+        bv = g.normal(size=(B, 3))
+        bv /= np.linalg.norm(bv, axis=1, keepdims=True)
+        cn = g.normal(size=3)
+        vn = g.normal(size=3)
+        vn /= np.linalg.norm(vn)
+        E, n, delta = 2.0, B + 2, 2
+        idx, score, count = oracle.retrieve(bc, bv, cn, vn, n, E, w_v, tau_c, cos_tau_v, delta, k)
+        R, t = _rotation(g), g.normal(size=3) * 10.0
+        idx2, score2, count2 = oracle.retrieve(bc @ R.T + t, bv @ R.T, R @ cn + t, R @ vn, n, E, w_v, tau_c, cos_tau_v,
+                                               delta, k)
+        # the motion changes scores and gate terms only by rounding; skip draws that sit on a
+        # gate threshold or have two candidates within rounding of each other
+        s, dist, dot = oracle.crc_oracle.retrieval_terms(bc, bv, cn, vn, E, w_v)
+        hyp.assume(np.all(np.abs(dist - tau_c) > 1e-9) and np.all(np.abs(dot - cos_tau_v) > 1e-9))
+        ss = np.sort(s)
+        hyp.assume(B < 2 or np.min(np.diff(ss)) > 1e-9)
+        assert count2 == count
+        assert list(idx2) == list(idx)
+        np.testing.assert_allclose(score2[:count], score[:count], rtol=1e-12, atol=1e-12)
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 2**31 - 1), h=st.integers(1, 4), w=st.integers(1, 5), F=st.integers(1, 3),
-       lam=st.floats(0.0, 4.0), sigma=st.floats(0.3, 3.0), a=st.floats(-3.0, 3.0), b=st.floats(-2.0, 2.0),
-       gaussian=st.booleans())
-def test_attention_affine_in_values_and_free_of_window_key_order(seed, h, w, F, lam, sigma, a, b, gaussian):
-    g = np.random.default_rng(seed)
-    Q, Kc, Vc, uv, valid, segs = _attn_case(g, h, w, F, 8)
-    form = "gaussian" if gaussian else "eq2"
-    O, lse = oracle.attention(Q, Kc, Vc, uv, valid, segs, h, w, F, lam, sigma, bias_form=form)
-    Oa, lsea = oracle.attention(Q, Kc, a * Vc + b, uv, valid, segs, h, w, F, lam, sigma, bias_form=form)
-    np.testing.assert_allclose(Oa, a * O + b, atol=1e-11)
-    np.testing.assert_array_equal(lsea, lse)  # the weights do not depend on the values
-    # window keys carry no bias: permuting them (K and V rows together) changes nothing
-    Nc = F * h * w
-    perm = np.arange(3 * Nc)
-    perm[2 * Nc:] = 2 * Nc + g.permutation(Nc)
-    Op, lsep = oracle.attention(Q, Kc[:, perm], Vc[:, perm], uv, valid, segs, h, w, F, lam, sigma, bias_form=form)
-    np.testing.assert_allclose(Op, O, atol=1e-12)
-    np.testing.assert_allclose(lsep, lse, atol=1e-12)
+    def _attn_case(g, h, w, F, d):
+        Nc = F * h * w
+        segs = [(0, Nc, oracle.crc_oracle.SEG_SINK, 0), (Nc, Nc, oracle.crc_oracle.SEG_RETRIEVED, 0),
+                (2 * Nc, Nc, oracle.crc_oracle.SEG_WINDOW, 0)]
+        Nk = 3 * Nc
+        Q = g.normal(size=(1, Nc, 1, d))
+        Kc = g.normal(size=(1, Nk, 1, d))
+        Vc = g.normal(size=(1, Nk, 1, d))
+        uv = g.uniform(-0.5, max(h, w), size=(Nc, F, 2))
+        valid = g.uniform(size=(Nc, F)) < 0.7
+        return Q, Kc, Vc, uv, valid, segs
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 2**31 - 1), d1=st.integers(-2000, 2000), d2=st.integers(-2000, 2000),
-       pairs=st.integers(1, 8), c0=st.integers(0, 3), theta=st.floats(10.0, 1e5), interleaved=st.booleans())
-def test_rope_reposition_group_law(seed, d1, d2, pairs, c0, theta, interleaved):
-    g = np.random.default_rng(seed)
-    c0 = 2 * c0  # the temporal block starts on an even channel
-    dim = c0 + 2 * pairs + 4
-    x = g.normal(size=(3, dim))
-    r = lambda y, dl: oracle.rope_reposition(y, dl, c0, pairs, theta, interleaved)  # noqa: E731
-    np.testing.assert_allclose(r(r(x, d1), d2), r(x, d1 + d2), atol=1e-9)
-    np.testing.assert_allclose(r(r(x, d1), -d1), x, atol=1e-9)
-    # each rotary pair keeps its norm; channels outside the block are untouched
-    y = r(x, d1)
-    if interleaved:
-        a0, a1 = slice(c0, c0 + 2 * pairs, 2), slice(c0 + 1, c0 + 2 * pairs, 2)
-    else:
-        a0, a1 = slice(c0, c0 + pairs), slice(c0 + pairs, c0 + 2 * pairs)
-    np.testing.assert_allclose(np.hypot(y[:, a0], y[:, a1]), np.hypot(x[:, a0], x[:, a1]), rtol=1e-12)
-    outside = np.r_[0:c0, c0 + 2 * pairs:dim]
-    np.testing.assert_array_equal(y[:, outside], x[:, outside])
-    assert math.isfinite(float(np.abs(y).max()))
+    @settings(**SETTINGS)
+    @given(seed=st.integers(0, 2**31 - 1), h=st.integers(1, 4), w=st.integers(1, 5), F=st.integers(1, 3),
+           lam=st.floats(0.0, 4.0), sigma=st.floats(0.3, 3.0), a=st.floats(-3.0, 3.0), b=st.floats(-2.0, 2.0),
+           gaussian=st.booleans())
+    def test_attention_affine_in_values_and_free_of_window_key_order(seed, h, w, F, lam, sigma, a, b, gaussian):
+        g = np.random.default_rng(seed)
+        Q, Kc, Vc, uv, valid, segs = _attn_case(g, h, w, F, 8)
+        form = "gaussian" if gaussian else "eq2"
+        O, lse = oracle.attention(Q, Kc, Vc, uv, valid, segs, h, w, F, lam, sigma, bias_form=form)
+        Oa, lsea = oracle.attention(Q, Kc, a * Vc + b, uv, valid, segs, h, w, F, lam, sigma, bias_form=form)
+        np.testing.assert_allclose(Oa, a * O + b, atol=1e-11)
+        np.testing.assert_array_equal(lsea, lse)  # the weights do not depend on the values
+        # window keys carry no bias: permuting them (K and V rows together) changes nothing
+        Nc = F * h * w
+        perm = np.arange(3 * Nc)
+        perm[2 * Nc:] = 2 * Nc + g.permutation(Nc)
+        Op, lsep = oracle.attention(Q, Kc[:, perm], Vc[:, perm], uv, valid, segs, h, w, F, lam, sigma, bias_form=form)
+        np.testing.assert_allclose(Op, O, atol=1e-12)
+        np.testing.assert_allclose(lsep, lse, atol=1e-12)
+
+
+    @settings(**SETTINGS)
+    @given(seed=st.integers(0, 2**31 - 1), d1=st.integers(-2000, 2000), d2=st.integers(-2000, 2000),
+           pairs=st.integers(1, 8), c0=st.integers(0, 3), theta=st.floats(10.0, 1e5), interleaved=st.booleans())
+    def test_rope_reposition_group_law(seed, d1, d2, pairs, c0, theta, interleaved):
+        g = np.random.default_rng(seed)
+        c0 = 2 * c0  # the temporal block starts on an even channel
+        dim = c0 + 2 * pairs + 4
+        x = g.normal(size=(3, dim))
+        r = lambda y, dl: oracle.rope_reposition(y, dl, c0, pairs, theta, interleaved)  # noqa: E731
+        np.testing.assert_allclose(r(r(x, d1), d2), r(x, d1 + d2), atol=1e-9)
+        np.testing.assert_allclose(r(r(x, d1), -d1), x, atol=1e-9)
+        # each rotary pair keeps its norm; channels outside the block are untouched
+        y = r(x, d1)
+        if interleaved:
+            a0, a1 = slice(c0, c0 + 2 * pairs, 2), slice(c0 + 1, c0 + 2 * pairs, 2)
+        else:
+            a0, a1 = slice(c0, c0 + pairs), slice(c0 + pairs, c0 + 2 * pairs)
+        np.testing.assert_allclose(np.hypot(y[:, a0], y[:, a1]), np.hypot(x[:, a0], x[:, a1]), rtol=1e-12)
+        outside = np.r_[0:c0, c0 + 2 * pairs:dim]
+        np.testing.assert_array_equal(y[:, outside], x[:, outside])
+        assert math.isfinite(float(np.abs(y).max()))
