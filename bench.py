@@ -732,6 +732,8 @@ def main():
         from paper_2607_21848_gb300.sweeps import correspond_sweep
 
         sweep = correspond_sweep(device)
+        sweep["iid_depth"] = {key: val for key, val in correspond_sweep(device, depth="iid").items()
+                              if key in ("ms", "gbs", "valid_fraction")}
         modes = opt_in_modes(W)
         stream_ctx = stream_context(device, rank_seed(rank))
         shapes = other_shapes(device, rank_seed(rank))
@@ -777,6 +779,9 @@ def main():
         line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path",
                            "correspond_sweep": sweep, "other_shapes": shapes, "opt_in_modes": modes,
                            "stream": stream_ctx}
+        if sweep is not None:
+            sweep["frac_of_hbm_peak"] = sweep["gbs"] / peaks["hbm"]
+            sweep["iid_depth"]["frac_of_hbm_peak"] = sweep["iid_depth"]["gbs"] / peaks["hbm"]
         for v in (shapes or {}).values():
             v["frac_of_bf16_peak"] = v["tflops"] / peaks["bf16_sus"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

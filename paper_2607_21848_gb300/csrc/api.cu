@@ -332,9 +332,6 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
   a.uv = d_uv;
   a.cell = d_cell;
   a.valid = d_valid;
-  a.div_S = crc::make_fastdiv((uint32_t)(k * shape->F));
-  a.div_hw = crc::make_fastdiv((uint32_t)(shape->h * shape->w));
-  a.div_w = crc::make_fastdiv((uint32_t)shape->w);
   cudaError_t e = crc::launch_correspond(a, s);
   return e == cudaSuccess ? CRC_OK : cuda_fail(e);
 }

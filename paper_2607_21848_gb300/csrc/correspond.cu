@@ -1,17 +1,18 @@
 // Depth-reprojection correspondence (Sec. 4.3, Eq. 3) with the occlusion-aware
 // visibility test (Eq. 4) and the exact-fallback rules of the design choices.
 //
-// One thread per (query token p, source frame s) pair, pairs laid out [N_q][S] so
-// that every output array is written fully coalesced.  At block start the
-// per-(target frame t, source frame s) transform
-//     A_ts = R_s^T R_t K_t^-1,   b_ts = R_s^T (c_t - c_s),   K_s
-// is composed from the current frames (kernel argument) and the bank records of
-// the retrieved chunk d_idx[r] (device memory, so no host round trip) and kept in
-// shared memory.  The composition runs in fp32 -- the per-pair arithmetic that
-// consumes it is fp32 anyway -- except for the camera-centre difference, which is
-// formed in fp64 so that nearby centres do not cancel; fp64 throughput on this GPU
-// is a small fraction of fp32's and every block repeats the composition.  Per pair:
-//     X_s = z_p A_ts (j, i, 1)^T + b_ts  (= Eq. 3's X_s),   u^ = pi(K_s X_s).
+// Pairs (query token p, source frame s) are laid out [N_q][S].  Per (target frame
+// t, source frame s) the kernel composes, at block start,
+//     M_ts = K_s R_s^T R_t K_t^-1,   m_ts = K_s R_s^T (c_t - c_s),
+// so that for a query at grid cell (j, i) with depth z
+//     K_s X_s = z M_ts (j, i, 1)^T + m_ts        (X_s of Eq. 3),
+// whose last component is [X_s]_z (K_s's last row is (0, 0, 1)), and
+//     u^ = pi(K_s X_s) = (first two components) / [X_s]_z.
+// The composition runs in fp32 -- the per-pair arithmetic that consumes it is fp32
+// anyway -- except for the camera-centre difference, formed in fp64 so that nearby
+// centres do not cancel.  The frame records are stored as fp64; their conversion to
+// fp32 runs on the integer pipe, since this GPU's fp64 and conversion throughput is
+// a small fraction of its fp32 and integer throughput and every block repeats it.
 #include <math.h>
 
 #include "internal.cuh"
@@ -23,14 +24,29 @@ namespace {
 constexpr int kMaxS = CRC_MAX_K * CRC_MAX_FRAMES;
 constexpr int kMaxPairs = CRC_MAX_FRAMES * kMaxS;
 
-// 24 words, 16-byte aligned, so that a pair's transform is six vector loads
+// 16 words, 16-byte aligned
 struct __align__(16) PairXf {
-  float A[9];
-  float b[3];
-  float Ks[9];
+  float M[9];     // M_ts = K_s A_ts, A_ts = R_s^T R_t K_t^-1; its last row is A_ts's
+  float m[3];     // m_ts = K_s b_ts, b_ts = R_s^T (c_t - c_s); NaN when the pair is not a retrieval, so that u^ is NaN
   int depth_off;  // offset of D_s in the bank depth array, -1 if the pair is not a retrieval
-  int pad[2];
+  int pad[3];
 };
+
+// IEEE-754 binary64 -> binary32, round to nearest even, on the integer pipe (this
+// GPU's fp64 and conversion rates are a small fraction of its integer rate).
+// Results below the binary32 normal range become signed zero.
+__device__ __forceinline__ float f64_to_f32(double x) {
+  const unsigned long long u = (unsigned long long)__double_as_longlong(x);
+  const unsigned sign = (unsigned)(u >> 32) & 0x80000000u;
+  const int e = (int)((u >> 52) & 0x7ff) - 1023 + 127;
+  if (e <= 0) return __uint_as_float(sign);
+  if (e >= 255) return __uint_as_float(sign | 0x7f800000u);
+  const unsigned long long mant = u & 0xfffffffffffffull;
+  unsigned r = ((unsigned)e << 23) | (unsigned)(mant >> 29);
+  const unsigned rest = (unsigned)(mant & 0x1fffffffull);
+  if (rest > 0x10000000u || (rest == 0x10000000u && (r & 1u))) ++r;  // a carry moves into the exponent
+  return __uint_as_float(sign | r);
+}
 
 __device__ void mat3_inverse(const float* m, float* inv) {
   const float c00 = m[4] * m[8] - m[5] * m[7];
@@ -51,153 +67,192 @@ __device__ void mat3_inverse(const float* m, float* inv) {
 
 }  // namespace
 
-__global__ void __launch_bounds__(256) correspond_kernel(const __grid_constant__ CorrespondArgs a) {
+// VIS: the visibility test of Eq. 4 is in force (eps finite).
+template <bool VIS>
+__global__ void __launch_bounds__(256, 5) correspond_kernel(const __grid_constant__ CorrespondArgs a, int FL) {
   __shared__ PairXf px[kMaxPairs];
+  __shared__ float src_KR[kMaxS][18];   // K_s, R_s
+  __shared__ double src_c[kMaxS][3];    // c_s
+  __shared__ int src_off[kMaxS];
+  __shared__ float tgt_RK[CRC_MAX_FRAMES][9];  // R_t K_t^-1
+  __shared__ double tgt_c[CRC_MAX_FRAMES][3];  // c_t
   const int S = a.k * a.F;
-  const int npairs = a.F * S;
   const int hw = a.h * a.w;
-  for (int q = threadIdx.x; q < npairs; q += blockDim.x) {
-    const int t = q / S, s = q - (q / S) * S;
-    const int r = s / a.F, f = s - (s / a.F) * a.F;
-    const int j = a.d_idx[r];
-    bool ok = (j >= 0) && (j < a.capacity);
-    if (a.d_count) ok = ok && (r < *a.d_count);
-    PairXf x;
-    x.pad[0] = x.pad[1] = 0;
-    if (ok) {
-      const double* ft = &a.cur.rec[t][0];
-      const double* fs = a.bank_frames + ((size_t)j * a.F + f) * kFrameDoubles;
-      float Kt[9], Rt[9], Rs[9], Ki[9], RK[9];
-      for (int e = 0; e < 9; ++e) {
-        Kt[e] = (float)ft[e];
-        Rt[e] = (float)ft[9 + e];
-        Rs[e] = (float)fs[9 + e];
+  const int Nq = a.F * hw;
+  const int R = blockDim.x / S;  // queries per block step
+  const int steps = ((Nq + R - 1) / R + gridDim.x - 1) / gridDim.x;
+  const int qb = blockIdx.x * steps * R;
+  const int q_end = min(Nq, qb + steps * R);
+  if (qb >= q_end) return;  // the whole block
+  const int t_lo = qb / hw, nt = (q_end - 1) / hw - t_lo + 1;
+
+  // The source values (21 per source frame) are loaded and converted by all threads
+  // but the first warp, a few each; meanwhile warp 0 forms R_t K_t^-1 for the block's
+  // target frames from the kernel arguments.
+  const int i = threadIdx.x;
+  if (i >= 32) {
+    for (int v = i - 32; v < S * kFrameDoubles; v += blockDim.x - 32) {
+      const int s = v / kFrameDoubles, e = v - s * kFrameDoubles;
+      const int r = s / a.F, f = s - r * a.F;
+      const int j = a.d_idx[r];
+      bool ok = (j >= 0) && (j < a.capacity);
+      if (a.d_count) ok = ok && (r < *a.d_count);
+      if (e == 0) src_off[s] = ok ? (int)(((size_t)j * a.F + f) * hw) : -1;
+      if (ok) {
+        const double x = a.bank_frames[((size_t)j * a.F + f) * kFrameDoubles + e];
+        if (e < 18)
+          src_KR[s][e] = f64_to_f32(x);
+        else
+          src_c[s][e - 18] = x;
       }
-      mat3_inverse(Kt, Ki);
-      for (int m = 0; m < 3; ++m)
-        for (int n = 0; n < 3; ++n) RK[3 * m + n] = Rt[3 * m + 0] * Ki[n] + Rt[3 * m + 1] * Ki[3 + n] + Rt[3 * m + 2] * Ki[6 + n];
-      // A = R_s^T (R_t K_t^-1)
-      for (int m = 0; m < 3; ++m)
-        for (int n = 0; n < 3; ++n) x.A[3 * m + n] = Rs[m] * RK[n] + Rs[3 + m] * RK[3 + n] + Rs[6 + m] * RK[6 + n];
-      const float dc[3] = {(float)(ft[18] - fs[18]), (float)(ft[19] - fs[19]), (float)(ft[20] - fs[20])};
-      for (int m = 0; m < 3; ++m) x.b[m] = Rs[m] * dc[0] + Rs[3 + m] * dc[1] + Rs[6 + m] * dc[2];
-      for (int e = 0; e < 9; ++e) x.Ks[e] = (float)fs[e];
-      x.depth_off = (int)(((size_t)j * a.F + f) * hw);
-    } else {
-      for (int e = 0; e < 9; ++e) x.A[e] = x.Ks[e] = 0.f;
-      x.b[0] = x.b[1] = x.b[2] = 0.f;
-      x.depth_off = -1;
     }
-    px[q] = x;
+  } else if (i < nt) {
+    const int t = t_lo + i;
+    const double* ft = &a.cur.rec[t][0];
+    float Kt[9], Rt[9], Ki[9];
+    for (int e = 0; e < 9; ++e) {
+      Kt[e] = f64_to_f32(ft[e]);
+      Rt[e] = f64_to_f32(ft[9 + e]);
+    }
+    mat3_inverse(Kt, Ki);
+    for (int m = 0; m < 3; ++m)
+      for (int n = 0; n < 3; ++n)
+        tgt_RK[i][3 * m + n] = Rt[3 * m + 0] * Ki[n] + Rt[3 * m + 1] * Ki[3 + n] + Rt[3 * m + 2] * Ki[6 + n];
+    for (int e = 0; e < 3; ++e) tgt_c[i][e] = ft[18 + e];
+  }
+  __syncthreads();
+  if (i < nt * S) {
+    const int tl = i / S, s = i - (i / S) * S;
+    PairXf x;
+    x.pad[0] = x.pad[1] = x.pad[2] = 0;
+    x.depth_off = src_off[s];
+    if (x.depth_off >= 0) {
+      const float* Ks = &src_KR[s][0];
+      const float* Rs = &src_KR[s][9];
+      const float* RK = &tgt_RK[tl][0];
+      float A[9], b[3];
+      // A = R_s^T (R_t K_t^-1), b = R_s^T (c_t - c_s) with the difference formed in fp64
+      for (int m = 0; m < 3; ++m)
+        for (int n = 0; n < 3; ++n) A[3 * m + n] = Rs[m] * RK[n] + Rs[3 + m] * RK[3 + n] + Rs[6 + m] * RK[6 + n];
+      float dc[3];
+      for (int e = 0; e < 3; ++e) dc[e] = f64_to_f32(tgt_c[tl][e] - src_c[s][e]);
+      for (int m = 0; m < 3; ++m) b[m] = Rs[m] * dc[0] + Rs[3 + m] * dc[1] + Rs[6 + m] * dc[2];
+      // M = K_s A and m = K_s b; the last rows are A's and b's
+      for (int m = 0; m < 2; ++m) {
+        for (int n = 0; n < 3; ++n) x.M[3 * m + n] = Ks[3 * m] * A[n] + Ks[3 * m + 1] * A[3 + n] + Ks[3 * m + 2] * A[6 + n];
+        x.m[m] = Ks[3 * m] * b[0] + Ks[3 * m + 1] * b[1] + Ks[3 * m + 2] * b[2];
+      }
+      for (int n = 0; n < 3; ++n) x.M[6 + n] = A[6 + n];
+      x.m[2] = b[2];
+    } else {
+      for (int e = 0; e < 9; ++e) x.M[e] = 0.f;
+      x.m[0] = x.m[1] = x.m[2] = __int_as_float(0x7fc00000);
+    }
+    px[i] = x;
   }
   __syncthreads();
 
-  const int total = a.F * hw * S;
-  const bool vis_test = !isinf(a.eps);
+  // Thread (g, qi, fi) handles source frame s = g FL + fi of queries qb + qi,
+  // qb + qi + R, ...: a warp covers 32 / FL adjacent queries x FL frames, so that
+  // its source-depth reads fall into few lines while each query's FL outputs stay
+  // contiguous.  A block step writes R S consecutive pairs.
+  const int fi = i % FL;
+  const int qi = (i / FL) % R;
+  const int s = (i / (FL * R)) * FL + fi;
+  int q = qb + qi;
+  if (q >= q_end) return;
+  int t = q / hw;
+  int iy = (q - t * hw) / a.w;
+  int jx = q - t * hw - iy * a.w;
+  float c0, c1, c2, r0, r1, r2, m0, m1, m2;
+  int doff;
+  {
+    const PairXf& x = px[(t - t_lo) * S + s];
+    c0 = x.M[0], c1 = x.M[3], c2 = x.M[6];
+    r0 = fmaf(x.M[1], (float)iy, x.M[2]);
+    r1 = fmaf(x.M[4], (float)iy, x.M[5]);
+    r2 = fmaf(x.M[7], (float)iy, x.M[8]);
+    m0 = x.m[0], m1 = x.m[1], m2 = x.m[2];
+    doff = x.depth_off;
+  }
   const float one_eps = 1.0f + a.eps;
-  // The block size is a multiple of S, so the grid stride is too and each thread
-  // keeps one source frame s for all its pairs.  Its transform for target frame t
-  // stays in registers and is reloaded only when t changes (at most F times).
-  // Each thread carries kILP pairs at once, so that their query-depth loads and
-  // then their source-depth gathers overlap in flight.
-  constexpr int kILP = 4;
-  const int stride = gridDim.x * blockDim.x;
-  const int first = blockIdx.x * blockDim.x + threadIdx.x;
-  const int s_own = first - (int)fastdiv((uint32_t)first, a.div_S) * S;
-  int t_cached = -1;
-  PairXf x;
-  for (int base = first; base < total; base += kILP * stride) {
-    int pr[kILP], tr[kILP], jx[kILP], iy[kILP];
-    float z[kILP];
-#pragma unroll
-    for (int u = 0; u < kILP; ++u) {
-      const int idx = base + u * stride;
-      pr[u] = idx < total ? (int)fastdiv((uint32_t)idx, a.div_S) : -1;
-      tr[u] = -1;
-      z[u] = 0.f;
-      if (pr[u] >= 0) {
-        tr[u] = (int)fastdiv((uint32_t)pr[u], a.div_hw);
-        const int rem = pr[u] - tr[u] * hw;
-        iy[u] = (int)fastdiv((uint32_t)rem, a.div_w);
-        jx[u] = rem - iy[u] * a.w;
-        z[u] = a.depth[pr[u]];
+  const float wf = (float)a.w, hf = (float)a.h;
+  size_t o = (size_t)q * S + s;
+  const size_t o_step = (size_t)R * S;
+  float z = a.depth[q];
+  for (; q < q_end; q += R, o += o_step) {
+    const float zn = q + R < q_end ? a.depth[q + R] : 0.f;  // next query's depth, in flight meanwhile
+    const float u0 = (float)jx;
+    // K_s X_s = z M (j, i, 1)^T + m; its last component is [X_s]_z
+    const float X0 = fmaf(z, fmaf(c0, u0, r0), m0);
+    const float X1 = fmaf(z, fmaf(c1, u0, r1), m1);
+    const float X2 = fmaf(z, fmaf(c2, u0, r2), m2);
+    float iq;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(iq) : "f"(X2));  // 1 ulp; a subnormal X2 gives inf, hence invalid
+    const float ux = X0 * iq, uy = X1 * iq;
+    const float vx = ux + 0.5f, vy = uy + 0.5f;
+    // the nearest cell is floor(u^ + 1/2); every comparison fails on NaN
+    bool ok = (z > 0.f) & (z < INFINITY) & (X2 > 0.f) & (X2 < INFINITY) & (vx >= 0.f) & (vx < wf) & (vy >= 0.f) &
+              (vy < hf);
+    int cell = ok ? __float2int_rd(vy) * a.w + __float2int_rd(vx) : -1;
+    if (VIS) {
+      const float ds = *(ok ? a.bank_depth + (doff + cell) : a.depth + q);
+      ok = ok & (X2 <= one_eps * ds);
+      cell = ok ? cell : -1;
+    }
+    reinterpret_cast<float2*>(a.uv)[o] = make_float2(ux, uy);
+    if (a.cell) a.cell[o] = cell;
+    a.valid[o] = ok ? 1 : 0;
+    jx += R;
+    if (jx >= a.w) {
+      const int t_was = t;
+      do {
+        jx -= a.w;
+        if (++iy == a.h) {
+          iy = 0;
+          ++t;
+        }
+      } while (jx >= a.w);
+      if (t < a.F) {
+        const PairXf& x = px[(t - t_lo) * S + s];
+        if (t != t_was) {
+          c0 = x.M[0], c1 = x.M[3], c2 = x.M[6];
+          m0 = x.m[0], m1 = x.m[1], m2 = x.m[2];
+          doff = x.depth_off;
+        }
+        r0 = fmaf(x.M[1], (float)iy, x.M[2]);
+        r1 = fmaf(x.M[4], (float)iy, x.M[5]);
+        r2 = fmaf(x.M[7], (float)iy, x.M[8]);
       }
     }
-    float ux[kILP], uy[kILP], X2[kILP];
-    int cell[kILP], doff[kILP];
-    bool valid[kILP];
-#pragma unroll
-    for (int u = 0; u < kILP; ++u) {
-      ux[u] = uy[u] = __int_as_float(0x7fc00000);  // NaN when the pair is not a retrieval
-      valid[u] = false;
-      cell[u] = -1;
-      X2[u] = 0.f;
-      doff[u] = -1;
-      if (pr[u] < 0) continue;
-      if (tr[u] != t_cached) {
-#pragma unroll
-        for (int v = 0; v < 6; ++v)
-          reinterpret_cast<float4*>(&x)[v] = reinterpret_cast<const float4*>(&px[tr[u] * S + s_own])[v];
-        t_cached = tr[u];
-      }
-      doff[u] = x.depth_off;
-      if (x.depth_off < 0) continue;
-      const float u0 = (float)jx[u], u1 = (float)iy[u];
-      const float a0 = x.A[0] * u0 + x.A[1] * u1 + x.A[2];
-      const float a1 = x.A[3] * u0 + x.A[4] * u1 + x.A[5];
-      const float a2 = x.A[6] * u0 + x.A[7] * u1 + x.A[8];
-      const float X0 = z[u] * a0 + x.b[0];
-      const float X1 = z[u] * a1 + x.b[1];
-      X2[u] = z[u] * a2 + x.b[2];
-      const float q0 = x.Ks[0] * X0 + x.Ks[1] * X1 + x.Ks[2] * X2[u];
-      const float q1 = x.Ks[3] * X0 + x.Ks[4] * X1 + x.Ks[5] * X2[u];
-      const float q2 = x.Ks[6] * X0 + x.Ks[7] * X1 + x.Ks[8] * X2[u];
-      const float iq = 1.0f / q2;  // one division: u^ within an ulp of q0 / q2
-      ux[u] = q0 * iq;
-      uy[u] = q1 * iq;
-      const float fx = floorf(ux[u] + 0.5f), fy = floorf(uy[u] + 0.5f);
-      valid[u] = isfinite(z[u]) && z[u] > 0.f && isfinite(ux[u]) && isfinite(uy[u]) && X2[u] > 0.f && fx >= 0.f &&
-                 fx < (float)a.w && fy >= 0.f && fy < (float)a.h;
-      if (valid[u]) cell[u] = (int)fy * a.w + (int)fx;
-    }
-    float ds[kILP];
-#pragma unroll
-    for (int u = 0; u < kILP; ++u)
-      ds[u] = (vis_test && valid[u]) ? a.bank_depth[doff[u] + cell[u]] : 0.f;
-#pragma unroll
-    for (int u = 0; u < kILP; ++u) {
-      if (pr[u] < 0) continue;
-      if (vis_test && valid[u] && !(X2[u] <= one_eps * ds[u])) {
-        valid[u] = false;
-        cell[u] = -1;
-      }
-      const int idx = base + u * stride;
-      reinterpret_cast<float2*>(a.uv)[idx] = make_float2(ux[u], uy[u]);
-      if (a.cell) a.cell[idx] = cell[u];
-      a.valid[idx] = valid[u] ? 1 : 0;
-    }
+    z = zn;
   }
 }
 
+template <bool VIS>
+static cudaError_t launch_v(const CorrespondArgs& a, cudaStream_t s, int sms, int S, int Nq) {
+  const int threads = (256 / S) * S;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel<VIS>, threads, 0) != cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  const int R = threads / S;
+  const int groups = (Nq + R - 1) / R;
+  const int blocks = groups < per_sm * sms ? groups : per_sm * sms;
+  int fl = 8;
+  while (S % fl != 0) --fl;  // frames per lane group: the largest divisor of S up to 8
+  correspond_kernel<VIS><<<blocks, threads, 0, s>>>(a, fl);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s) {
-  const int total = a.F * a.h * a.w * a.k * a.F;
-  if (total == 0) return cudaSuccess;
+  const int Nq = a.F * a.h * a.w;
+  const int S = a.k * a.F;
+  if (Nq == 0 || S == 0) return cudaSuccess;
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // grid-stride over the pairs with four pairs in flight per thread: one resident
-  // wave, so that each block's composition of the transforms is amortised over
-  // many pairs
-  const int S = a.k * a.F;
-  const int threads = (256 / S) * S;  // a multiple of S (S <= 32)
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel, threads, 0) != cudaSuccess ||
-      per_sm < 1)
-    per_sm = 1;
-  int blocks = (total + 4 * threads - 1) / (4 * threads);
-  if (blocks > per_sm * sms) blocks = per_sm * sms;
-  correspond_kernel<<<blocks, threads, 0, s>>>(a);
-  return cudaGetLastError();
+  return isinf(a.eps) ? launch_v<false>(a, s, sms, S, Nq) : launch_v<true>(a, s, sms, S, Nq);
 }
 
 }  // namespace crc

@@ -121,23 +121,6 @@ struct GatherOnlyArgs {
 };
 cudaError_t launch_gather(const GatherOnlyArgs& a, cudaStream_t s);
 
-// Division of unsigned 32-bit n by an invariant divisor d >= 1 (Granlund and
-// Montgomery, "Division by invariant integers using multiplication", 1994):
-// with l = ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1, the quotient is
-// (mulhi(m, n) + n) >> l, the sum formed in 64 bits.  Exact for every n < 2^32.
-struct FastDiv {
-  uint32_t d, m, l;
-};
-inline FastDiv make_fastdiv(uint32_t d) {
-  uint32_t l = 0;
-  while (l < 32 && (1ull << l) < d) ++l;
-  const uint64_t m = (((1ull << 32) * ((1ull << l) - d)) / d) + 1;
-  return FastDiv{d, (uint32_t)m, l};
-}
-__device__ __forceinline__ uint32_t fastdiv(uint32_t n, const FastDiv& f) {
-  return (uint32_t)(((uint64_t)__umulhi(f.m, n) + n) >> f.l);
-}
-
 struct CorrespondArgs {
   FrameSet cur;
   const float* depth;        // [F][h][w]
@@ -151,7 +134,6 @@ struct CorrespondArgs {
   float* uv;
   int32_t* cell;             // may be null
   uint8_t* valid;
-  FastDiv div_S, div_hw, div_w;  // k*F, h*w, w
 };
 cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s);
 

@@ -1,6 +1,7 @@
 """Stand-alone sweeps of single kernels, for measurement and profiling (e.g. under ncu):
 
-  python -m paper_2607_21848_gb300.sweeps correspond   # 126 MB reprojection sweep
+  python -m paper_2607_21848_gb300.sweeps correspond      # 126 MB reprojection sweep, scene depth
+  python -m paper_2607_21848_gb300.sweeps correspond-iid  # the same with depth drawn per token
   python -m paper_2607_21848_gb300.sweeps gather       # crc_gather, plain and re-positioned
 """
 
@@ -10,26 +11,44 @@ import json
 import sys
 
 
-def correspond_sweep(device="cuda:0", iters: int = 10):
+def correspond_sweep(device="cuda:0", iters: int = 20, depth: str = "scene"):
     """Reprojection (Eq. 3-4) at a scale where it is no longer launch-bound: 4 frames of
     180 x 320 tokens (230400 queries) against 8 retrieved chunks (32 source frames),
-    7.4 M (query, frame) pairs and 126 MB in one launch.  A sweep, not a configuration."""
+    7.4 M (query, frame) pairs and 126 MB in one launch.  A sweep, not a configuration.
+
+    depth="scene": the chunks are 9 consecutive chunks of a ground random walk through
+    a room of walls and boards (the scene model of the synthetic workloads), and every
+    depth map is rendered from that scene, so depth is piecewise smooth as in real
+    footage.  depth="iid": depth drawn independently per token, log-uniform on
+    [0.5, 20]; neighbouring tokens then land in unrelated cells of every source map,
+    the worst case for the source-depth reads of the visibility test."""
     import math
 
+    import numpy as np
     import torch
 
     import synth
+    from synth import workloads as W
     from paper_2607_21848_gb300 import api
 
     F, h, w, k = 4, 180, 320, 8
     K = synth.pinhole(h, w, 90.0)
-    fr = synth.random_walk(synth.rng(999, "sweep"), k + 1, F, K)
+    fr = synth.random_walk(synth.rng(999, "sweep"), k + 1, F, K, step=0.5, radius=24.0)
     bank = api.Bank(k + 1, F, h, w, 1, 1, 64, torch.float32, 1, device=device, with_kv=False)
     shp = api.shape(1, 1, 64, F, h, w, torch.float32)
     api.crc_bank_insert_poses(bank, shp, 0, synth.frame_records(fr))
-    g = torch.Generator(device=device).manual_seed(99)
-    bank.depth.copy_(torch.exp(torch.rand(bank.depth.shape, generator=g, device=device) * math.log(40.0)) * 0.5)
-    depth = bank.depth[k].clone()
+    if depth == "scene":
+        scene = W.Scene.room(synth.rng(999, "scene"), radius=40.0, n_walls=12, n_boards=60, board_rmin=2.0,
+                             board_rmax=36.0)
+        dep = np.stack([np.stack([W.render_depth(scene, fr.K[j, f], fr.R[j, f], fr.c[j, f], h, w, 0.5, 50.0)
+                                  for f in range(F)]) for j in range(k + 1)]).astype(np.float32)
+        bank.depth.copy_(torch.from_numpy(dep).to(device))
+    elif depth == "iid":
+        g = torch.Generator(device=device).manual_seed(99)
+        bank.depth.copy_(torch.exp(torch.rand(bank.depth.shape, generator=g, device=device) * math.log(40.0)) * 0.5)
+    else:
+        raise ValueError(f"unknown depth model {depth!r}")
+    depth_cur = bank.depth[k].clone()
     idx = torch.arange(k, dtype=torch.int32, device=device)
     count = torch.full((1,), k, dtype=torch.int32, device=device)
     Nq, S = F * h * w, k * F
@@ -39,7 +58,7 @@ def correspond_sweep(device="cuda:0", iters: int = 10):
     cur = synth.frame_records(fr[k])
 
     def run():
-        api.crc_correspond(shp, cur, depth, bank, idx, count, k, 0.05, uv, cell, valid)
+        api.crc_correspond(shp, cur, depth_cur, bank, idx, count, k, 0.05, uv, cell, valid)
 
     run()
     torch.cuda.synchronize()
@@ -52,7 +71,7 @@ def correspond_sweep(device="cuda:0", iters: int = 10):
     torch.cuda.synchronize()
     t = e0.elapsed_time(e1) / 1e3 / iters
     nbytes = Nq * 4 + Nq * S * (8 + 4 + 1 + 4)
-    return {"queries": Nq, "source_frames": S, "pairs": Nq * S, "bytes": nbytes, "ms": t * 1e3,
+    return {"depth": depth, "queries": Nq, "source_frames": S, "pairs": Nq * S, "bytes": nbytes, "ms": t * 1e3,
             "gbs": nbytes / t / 1e9, "valid_fraction": float(valid.float().mean())}
 
 
@@ -101,6 +120,8 @@ def main(argv=None):
     build.build()
     if what == "correspond":
         print(json.dumps(correspond_sweep("cuda:0")))
+    elif what == "correspond-iid":
+        print(json.dumps(correspond_sweep("cuda:0", depth="iid")))
     elif what == "gather":
         print(json.dumps(gather_sweep("cuda:0")))
     else:
