@@ -733,7 +733,7 @@ def main():
 
         sweep = correspond_sweep(device)
         sweep["iid_depth"] = {key: val for key, val in correspond_sweep(device, depth="iid").items()
-                              if key in ("ms", "gbs", "valid_fraction")}
+                              if key in ("ms", "gbs", "eager_ms", "valid_fraction")}
         modes = opt_in_modes(W)
         stream_ctx = stream_context(device, rank_seed(rank))
         shapes = other_shapes(device, rank_seed(rank))

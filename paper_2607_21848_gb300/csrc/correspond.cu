@@ -48,6 +48,31 @@ __device__ __forceinline__ float f64_to_f32(double x) {
   return __uint_as_float(sign | r);
 }
 
+// packed fp32 pairs (f32x2 ALU ops): each lane rounds exactly as the scalar op does
+__device__ __forceinline__ uint64_t pk2(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 __device__ void mat3_inverse(const float* m, float* inv) {
   const float c00 = m[4] * m[8] - m[5] * m[7];
   const float c01 = m[5] * m[6] - m[3] * m[8];
@@ -67,9 +92,10 @@ __device__ void mat3_inverse(const float* m, float* inv) {
 
 }  // namespace
 
-// VIS: the visibility test of Eq. 4 is in force (eps finite).
-template <bool VIS>
-__global__ void __launch_bounds__(256, 5) correspond_kernel(const __grid_constant__ CorrespondArgs a, int FL) {
+// VIS: the visibility test of Eq. 4 is in force (eps finite).  P: source frames per
+// thread (2 when S is even and the outputs are aligned for 16-byte stores).
+template <int P, bool VIS, typename Idx>
+__global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constant__ CorrespondArgs a, int FL) {
   __shared__ PairXf px[kMaxPairs];
   __shared__ float src_KR[kMaxS][18];   // K_s, R_s
   __shared__ double src_c[kMaxS][3];    // c_s
@@ -79,7 +105,8 @@ __global__ void __launch_bounds__(256, 5) correspond_kernel(const __grid_constan
   const int S = a.k * a.F;
   const int hw = a.h * a.w;
   const int Nq = a.F * hw;
-  const int R = blockDim.x / S;  // queries per block step
+  const int L = S / P;           // threads per query
+  const int R = blockDim.x / L;  // queries per block step
   const int steps = ((Nq + R - 1) / R + gridDim.x - 1) / gridDim.x;
   const int qb = blockIdx.x * steps * R;
   const int q_end = min(Nq, qb + steps * R);
@@ -152,57 +179,92 @@ __global__ void __launch_bounds__(256, 5) correspond_kernel(const __grid_constan
   }
   __syncthreads();
 
-  // Thread (g, qi, fi) handles source frame s = g FL + fi of queries qb + qi,
-  // qb + qi + R, ...: a warp covers 32 / FL adjacent queries x FL frames, so that
-  // its source-depth reads fall into few lines while each query's FL outputs stay
-  // contiguous.  A block step writes R S consecutive pairs.
-  const int fi = i % FL;
-  const int qi = (i / FL) % R;
-  const int s = (i / (FL * R)) * FL + fi;
+  // Thread (g, qi, fi) handles source frames s0 = g FL + P fi .. s0 + P - 1 of
+  // queries qb + qi, qb + qi + R, ...: a warp covers 32 P / FL adjacent queries x FL
+  // frames, so that its source-depth reads fall into few lines while each query's FL
+  // outputs stay contiguous.  A block step writes R S consecutive pairs.
+  const int FLP = FL / P;
+  const int fi = i % FLP;
+  const int qi = (i / FLP) % R;
+  const int s0 = (i / (FLP * R)) * FL + fi * P;
   int q = qb + qi;
   if (q >= q_end) return;
   int t = q / hw;
   int iy = (q - t * hw) / a.w;
   int jx = q - t * hw - iy * a.w;
-  float c0, c1, c2, r0, r1, r2, m0, m1, m2;
-  int doff;
-  {
-    const PairXf& x = px[(t - t_lo) * S + s];
-    c0 = x.M[0], c1 = x.M[3], c2 = x.M[6];
-    r0 = fmaf(x.M[1], (float)iy, x.M[2]);
-    r1 = fmaf(x.M[4], (float)iy, x.M[5]);
-    r2 = fmaf(x.M[7], (float)iy, x.M[8]);
-    m0 = x.m[0], m1 = x.m[1], m2 = x.m[2];
-    doff = x.depth_off;
+  // the (t, s) transforms of the thread's P frames, lane p of each packed pair for s0 + p
+  float c0[P], c1[P], c2[P], r0[P], r1[P], r2[P], m0[P], m1[P], m2[P];
+  int doff[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    const PairXf& x = px[(t - t_lo) * S + s0 + p];
+    c0[p] = x.M[0], c1[p] = x.M[3], c2[p] = x.M[6];
+    r0[p] = fmaf(x.M[1], (float)iy, x.M[2]);
+    r1[p] = fmaf(x.M[4], (float)iy, x.M[5]);
+    r2[p] = fmaf(x.M[7], (float)iy, x.M[8]);
+    m0[p] = x.m[0], m1[p] = x.m[1], m2[p] = x.m[2];
+    doff[p] = x.depth_off;
   }
   const float one_eps = 1.0f + a.eps;
   const float wf = (float)a.w, hf = (float)a.h;
-  size_t o = (size_t)q * S + s;
-  const size_t o_step = (size_t)R * S;
+  Idx o = (Idx)q * (Idx)S + (Idx)s0;
+  const Idx o_step = (Idx)R * (Idx)S;
   float z = a.depth[q];
   for (; q < q_end; q += R, o += o_step) {
     const float zn = q + R < q_end ? a.depth[q + R] : 0.f;  // next query's depth, in flight meanwhile
     const float u0 = (float)jx;
-    // K_s X_s = z M (j, i, 1)^T + m; its last component is [X_s]_z
-    const float X0 = fmaf(z, fmaf(c0, u0, r0), m0);
-    const float X1 = fmaf(z, fmaf(c1, u0, r1), m1);
-    const float X2 = fmaf(z, fmaf(c2, u0, r2), m2);
-    float iq;
-    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(iq) : "f"(X2));  // 1 ulp; a subnormal X2 gives inf, hence invalid
-    const float ux = X0 * iq, uy = X1 * iq;
-    const float vx = ux + 0.5f, vy = uy + 0.5f;
-    // the nearest cell is floor(u^ + 1/2); every comparison fails on NaN
-    bool ok = (z > 0.f) & (z < INFINITY) & (X2 > 0.f) & (X2 < INFINITY) & (vx >= 0.f) & (vx < wf) & (vy >= 0.f) &
-              (vy < hf);
-    int cell = ok ? __float2int_rd(vy) * a.w + __float2int_rd(vx) : -1;
-    if (VIS) {
-      const float ds = *(ok ? a.bank_depth + (doff + cell) : a.depth + q);
-      ok = ok & (X2 <= one_eps * ds);
-      cell = ok ? cell : -1;
+    const bool z_ok = (z > 0.f) & (z < INFINITY);
+    float ux[P], uy[P], X2[P];
+    if (P == 2) {
+      // K_s X_s = z M (j, i, 1)^T + m for both frames at once; its last component is [X_s]_z
+      const uint64_t U0 = pk2(u0, u0), Z = pk2(z, z);
+      const uint64_t X0 = ffma2(Z, ffma2(pk2(c0[0], c0[P - 1]), U0, pk2(r0[0], r0[P - 1])), pk2(m0[0], m0[P - 1]));
+      const uint64_t X1 = ffma2(Z, ffma2(pk2(c1[0], c1[P - 1]), U0, pk2(r1[0], r1[P - 1])), pk2(m1[0], m1[P - 1]));
+      const uint64_t XZ = ffma2(Z, ffma2(pk2(c2[0], c2[P - 1]), U0, pk2(r2[0], r2[P - 1])), pk2(m2[0], m2[P - 1]));
+      upk2(XZ, X2[0], X2[P - 1]);
+      float iq0, iq1;
+      asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(iq0) : "f"(X2[0]));
+      asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(iq1) : "f"(X2[P - 1]));
+      const uint64_t IQ = pk2(iq0, iq1);
+      upk2(fmul2(X0, IQ), ux[0], ux[P - 1]);
+      upk2(fmul2(X1, IQ), uy[0], uy[P - 1]);
+    } else {
+      const float X0 = fmaf(z, fmaf(c0[0], u0, r0[0]), m0[0]);
+      const float X1 = fmaf(z, fmaf(c1[0], u0, r1[0]), m1[0]);
+      X2[0] = fmaf(z, fmaf(c2[0], u0, r2[0]), m2[0]);
+      float iq;
+      asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(iq) : "f"(X2[0]));  // 1 ulp; a subnormal X2 gives inf, hence invalid
+      ux[0] = X0 * iq;
+      uy[0] = X1 * iq;
     }
-    reinterpret_cast<float2*>(a.uv)[o] = make_float2(ux, uy);
-    if (a.cell) a.cell[o] = cell;
-    a.valid[o] = ok ? 1 : 0;
+    bool ok[P];
+    int cell[P];
+#pragma unroll
+    for (int p = 0; p < P; ++p) {
+      const float vx = ux[p] + 0.5f, vy = uy[p] + 0.5f;
+      // the nearest cell is floor(u^ + 1/2); every comparison fails on NaN
+      ok[p] = z_ok & (X2[p] > 0.f) & (X2[p] < INFINITY) & (vx >= 0.f) & (vx < wf) & (vy >= 0.f) & (vy < hf);
+      cell[p] = ok[p] ? __float2int_rd(vy) * a.w + __float2int_rd(vx) : -1;
+    }
+    if (VIS) {
+      float ds[P];
+#pragma unroll
+      for (int p = 0; p < P; ++p) ds[p] = *(ok[p] ? a.bank_depth + (doff[p] + cell[p]) : a.depth + q);
+#pragma unroll
+      for (int p = 0; p < P; ++p) {
+        ok[p] = ok[p] & (X2[p] <= one_eps * ds[p]);
+        cell[p] = ok[p] ? cell[p] : -1;
+      }
+    }
+    if (P == 2) {
+      *reinterpret_cast<float4*>(a.uv + 2 * o) = make_float4(ux[0], uy[0], ux[P - 1], uy[P - 1]);
+      if (a.cell) *reinterpret_cast<int2*>(a.cell + o) = make_int2(cell[0], cell[P - 1]);
+      *reinterpret_cast<uint16_t*>(a.valid + o) = (uint16_t)((ok[0] ? 1u : 0u) | (ok[P - 1] ? 0x100u : 0u));
+    } else {
+      reinterpret_cast<float2*>(a.uv)[o] = make_float2(ux[0], uy[0]);
+      if (a.cell) a.cell[o] = cell[0];
+      a.valid[o] = ok[0] ? 1 : 0;
+    }
     jx += R;
     if (jx >= a.w) {
       const int t_was = t;
@@ -214,35 +276,45 @@ __global__ void __launch_bounds__(256, 5) correspond_kernel(const __grid_constan
         }
       } while (jx >= a.w);
       if (t < a.F) {
-        const PairXf& x = px[(t - t_lo) * S + s];
-        if (t != t_was) {
-          c0 = x.M[0], c1 = x.M[3], c2 = x.M[6];
-          m0 = x.m[0], m1 = x.m[1], m2 = x.m[2];
-          doff = x.depth_off;
+#pragma unroll
+        for (int p = 0; p < P; ++p) {
+          const PairXf& x = px[(t - t_lo) * S + s0 + p];
+          if (t != t_was) {
+            c0[p] = x.M[0], c1[p] = x.M[3], c2[p] = x.M[6];
+            m0[p] = x.m[0], m1[p] = x.m[1], m2[p] = x.m[2];
+            doff[p] = x.depth_off;
+          }
+          r0[p] = fmaf(x.M[1], (float)iy, x.M[2]);
+          r1[p] = fmaf(x.M[4], (float)iy, x.M[5]);
+          r2[p] = fmaf(x.M[7], (float)iy, x.M[8]);
         }
-        r0 = fmaf(x.M[1], (float)iy, x.M[2]);
-        r1 = fmaf(x.M[4], (float)iy, x.M[5]);
-        r2 = fmaf(x.M[7], (float)iy, x.M[8]);
       }
     }
     z = zn;
   }
 }
 
-template <bool VIS>
+template <int P, bool VIS, typename Idx>
 static cudaError_t launch_v(const CorrespondArgs& a, cudaStream_t s, int sms, int S, int Nq) {
-  const int threads = (256 / S) * S;
+  const int L = S / P;
+  const int threads = (256 / L) * L;
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel<VIS>, threads, 0) != cudaSuccess ||
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, correspond_kernel<P, VIS, Idx>, threads, 0) !=
+          cudaSuccess ||
       per_sm < 1)
     per_sm = 1;
-  const int R = threads / S;
+  const int R = threads / L;
   const int groups = (Nq + R - 1) / R;
   const int blocks = groups < per_sm * sms ? groups : per_sm * sms;
   int fl = 8;
-  while (S % fl != 0) --fl;  // frames per lane group: the largest divisor of S up to 8
-  correspond_kernel<VIS><<<blocks, threads, 0, s>>>(a, fl);
+  while (S % fl != 0 || fl % P != 0) --fl;  // frames per lane group: the largest divisor of S up to 8 (a multiple of P)
+  correspond_kernel<P, VIS, Idx><<<blocks, threads, 0, s>>>(a, fl);
   return cudaGetLastError();
+}
+
+template <int P, typename Idx>
+static cudaError_t launch_pi(const CorrespondArgs& a, cudaStream_t s, int sms, int S, int Nq) {
+  return isinf(a.eps) ? launch_v<P, false, Idx>(a, s, sms, S, Nq) : launch_v<P, true, Idx>(a, s, sms, S, Nq);
 }
 
 cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s) {
@@ -252,7 +324,13 @@ cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  return isinf(a.eps) ? launch_v<false>(a, s, sms, S, Nq) : launch_v<true>(a, s, sms, S, Nq);
+  // two source frames per thread when S is even and the outputs take 16-, 8- and 2-byte stores
+  const bool two = S % 2 == 0 && ((uintptr_t)a.uv & 15) == 0 && ((uintptr_t)a.cell & 7) == 0 &&
+                   ((uintptr_t)a.valid & 1) == 0;
+  const bool narrow = (uint64_t)Nq * (uint64_t)S < (1ull << 32);  // pair offsets fit 32 bits
+  if (two)
+    return narrow ? launch_pi<2, uint32_t>(a, s, sms, S, Nq) : launch_pi<2, size_t>(a, s, sms, S, Nq);
+  return narrow ? launch_pi<1, uint32_t>(a, s, sms, S, Nq) : launch_pi<1, size_t>(a, s, sms, S, Nq);
 }
 
 }  // namespace crc
