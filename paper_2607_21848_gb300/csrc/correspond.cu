@@ -13,6 +13,12 @@
 // centres do not cancel.  The frame records are stored as fp64; their conversion to
 // fp32 runs on the integer pipe, since this GPU's fp64 and conversion throughput is
 // a small fraction of its fp32 and integer throughput and every block repeats it.
+//
+// The launch allows programmatic stream serialization: a block first does the work
+// that depends on its arguments alone, then waits for the grid before it
+// (griddepcontrol.wait) before it reads bank data or depths or writes an output, and
+// once its prologue is done it lets the next grid begin its launch, so that launch
+// latency overlaps the running grid.
 #include <math.h>
 
 #include "internal.cuh"
@@ -113,10 +119,27 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   if (qb >= q_end) return;  // the whole block
   const int t_lo = qb / hw, nt = (q_end - 1) / hw - t_lo + 1;
 
-  // The source values (21 per source frame) are loaded and converted by all threads
-  // but the first warp, a few each; meanwhile warp 0 forms R_t K_t^-1 for the block's
-  // target frames from the kernel arguments.
+  // Warp 0 forms R_t K_t^-1 for the block's target frames from the kernel arguments
+  // alone, before the wait on the grid this launch depends on; everything below reads
+  // data that grid may write (indices, bank records, depths) or writes outputs.
   const int i = threadIdx.x;
+  if (i < nt) {
+    const int t = t_lo + i;
+    const double* ft = &a.cur.rec[t][0];
+    float Kt[9], Rt[9], Ki[9];
+    for (int e = 0; e < 9; ++e) {
+      Kt[e] = f64_to_f32(ft[e]);
+      Rt[e] = f64_to_f32(ft[9 + e]);
+    }
+    mat3_inverse(Kt, Ki);
+    for (int m = 0; m < 3; ++m)
+      for (int n = 0; n < 3; ++n)
+        tgt_RK[i][3 * m + n] = Rt[3 * m + 0] * Ki[n] + Rt[3 * m + 1] * Ki[3 + n] + Rt[3 * m + 2] * Ki[6 + n];
+    for (int e = 0; e < 3; ++e) tgt_c[i][e] = ft[18 + e];
+  }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // The source values (21 per source frame) are loaded and converted by all threads
+  // but the first warp, a few each.
   if (i >= 32) {
     for (int v = i - 32; v < S * kFrameDoubles; v += blockDim.x - 32) {
       const int s = v / kFrameDoubles, e = v - s * kFrameDoubles;
@@ -133,19 +156,6 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
           src_c[s][e - 18] = x;
       }
     }
-  } else if (i < nt) {
-    const int t = t_lo + i;
-    const double* ft = &a.cur.rec[t][0];
-    float Kt[9], Rt[9], Ki[9];
-    for (int e = 0; e < 9; ++e) {
-      Kt[e] = f64_to_f32(ft[e]);
-      Rt[e] = f64_to_f32(ft[9 + e]);
-    }
-    mat3_inverse(Kt, Ki);
-    for (int m = 0; m < 3; ++m)
-      for (int n = 0; n < 3; ++n)
-        tgt_RK[i][3 * m + n] = Rt[3 * m + 0] * Ki[n] + Rt[3 * m + 1] * Ki[3 + n] + Rt[3 * m + 2] * Ki[6 + n];
-    for (int e = 0; e < 3; ++e) tgt_c[i][e] = ft[18 + e];
   }
   __syncthreads();
   if (i < nt * S) {
@@ -179,6 +189,7 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   }
   __syncthreads();
 
+  asm volatile("griddepcontrol.launch_dependents;");  // the next grid may begin its launch
   // Thread (g, qi, fi) handles source frames s0 = g FL + P fi .. s0 + P - 1 of
   // queries qb + qi, qb + qi + R, ...: a warp covers 32 P / FL adjacent queries x FL
   // frames, so that its source-depth reads fall into few lines while each query's FL
@@ -308,8 +319,17 @@ static cudaError_t launch_v(const CorrespondArgs& a, cudaStream_t s, int sms, in
   const int blocks = groups < per_sm * sms ? groups : per_sm * sms;
   int fl = 8;
   while (S % fl != 0 || fl % P != 0) --fl;  // frames per lane group: the largest divisor of S up to 8 (a multiple of P)
-  correspond_kernel<P, VIS, Idx><<<blocks, threads, 0, s>>>(a, fl);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(blocks);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, correspond_kernel<P, VIS, Idx>, a, fl);
 }
 
 template <int P, typename Idx>
