@@ -29,6 +29,9 @@ namespace {
 
 constexpr int kMaxS = CRC_MAX_K * CRC_MAX_FRAMES;
 constexpr int kMaxPairs = CRC_MAX_FRAMES * kMaxS;
+// frame values loaded per prologue thread: 4 (256 - 31 - 32) >= 21 kMaxS
+constexpr int kLoadsPerThread = 4;
+static_assert(kLoadsPerThread * (256 - 31 - 32) >= kFrameDoubles * kMaxS, "prologue loads do not cover the records");
 
 // 16 words, 16-byte aligned
 struct __align__(16) PairXf {
@@ -73,11 +76,6 @@ __device__ __forceinline__ uint64_t fmul2(uint64_t a, uint64_t b) {
   asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
-__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
 
 __device__ void mat3_inverse(const float* m, float* inv) {
   const float c00 = m[4] * m[8] - m[5] * m[7];
@@ -118,11 +116,20 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   const int q_end = min(Nq, qb + steps * R);
   if (qb >= q_end) return;  // the whole block
   const int t_lo = qb / hw, nt = (q_end - 1) / hw - t_lo + 1;
+  // Thread (g, qi, fi) handles source frames s0 = g FL + P fi .. s0 + P - 1 of
+  // queries qb + qi, qb + qi + R, ...: a warp covers 32 P / FL adjacent queries x FL
+  // frames, so that its source-depth reads fall into few lines while each query's FL
+  // outputs stay contiguous.  A block step writes R S consecutive pairs.
+  const int i = threadIdx.x;
+  const int FLP = FL / P;
+  const int fi = i % FLP;
+  const int qi = (i / FLP) % R;
+  const int s0 = (i / (FLP * R)) * FL + fi * P;
+  int q = qb + qi;
 
   // Warp 0 forms R_t K_t^-1 for the block's target frames from the kernel arguments
   // alone, before the wait on the grid this launch depends on; everything below reads
   // data that grid may write (indices, bank records, depths) or writes outputs.
-  const int i = threadIdx.x;
   if (i < nt) {
     const int t = t_lo + i;
     const double* ft = &a.cur.rec[t][0];
@@ -138,22 +145,44 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
     for (int e = 0; e < 3; ++e) tgt_c[i][e] = ft[18 + e];
   }
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  float z = q < q_end ? a.depth[q] : 0.f;  // the first query's depth, in flight through the prologue
   // The source values (21 per source frame) are loaded and converted by all threads
-  // but the first warp, a few each.
+  // but the first warp, in two rounds of independent loads: the slot indices, then
+  // the records.  A block has at least 256 - 31 threads (a multiple of S / P <= 32),
+  // so kLoadsPerThread loads per thread cover the 21 S <= 672 values.
   if (i >= 32) {
-    for (int v = i - 32; v < S * kFrameDoubles; v += blockDim.x - 32) {
-      const int s = v / kFrameDoubles, e = v - s * kFrameDoubles;
-      const int r = s / a.F, f = s - r * a.F;
-      const int j = a.d_idx[r];
-      bool ok = (j >= 0) && (j < a.capacity);
-      if (a.d_count) ok = ok && (r < *a.d_count);
-      if (e == 0) src_off[s] = ok ? (int)(((size_t)j * a.F + f) * hw) : -1;
-      if (ok) {
-        const double x = a.bank_frames[((size_t)j * a.F + f) * kFrameDoubles + e];
+    const int nthr = blockDim.x - 32;
+    const int nv = S * kFrameDoubles;
+    const int cnt = a.d_count ? *a.d_count : CRC_MAX_K;
+    int jr[kLoadsPerThread];
+#pragma unroll
+    for (int u = 0; u < kLoadsPerThread; ++u) {
+      const int v = i - 32 + u * nthr;
+      jr[u] = v < nv ? a.d_idx[(v / kFrameDoubles) / a.F] : -1;
+    }
+    double xv[kLoadsPerThread];
+#pragma unroll
+    for (int u = 0; u < kLoadsPerThread; ++u) {
+      const int v = i - 32 + u * nthr;
+      xv[u] = 0.0;
+      if (v < nv) {
+        const int s = v / kFrameDoubles, e = v - s * kFrameDoubles;
+        const int r = s / a.F, f = s - r * a.F;
+        const int j = jr[u];
+        const bool ok = (j >= 0) && (j < a.capacity) && (r < cnt);
+        if (e == 0) src_off[s] = ok ? (int)(((size_t)j * a.F + f) * hw) : -1;
+        if (ok) xv[u] = a.bank_frames[((size_t)j * a.F + f) * kFrameDoubles + e];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kLoadsPerThread; ++u) {
+      const int v = i - 32 + u * nthr;
+      if (v < nv) {
+        const int s = v / kFrameDoubles, e = v - s * kFrameDoubles;
         if (e < 18)
-          src_KR[s][e] = f64_to_f32(x);
+          src_KR[s][e] = f64_to_f32(xv[u]);
         else
-          src_c[s][e - 18] = x;
+          src_c[s][e - 18] = xv[u];
       }
     }
   }
@@ -190,15 +219,6 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   __syncthreads();
 
   asm volatile("griddepcontrol.launch_dependents;");  // the next grid may begin its launch
-  // Thread (g, qi, fi) handles source frames s0 = g FL + P fi .. s0 + P - 1 of
-  // queries qb + qi, qb + qi + R, ...: a warp covers 32 P / FL adjacent queries x FL
-  // frames, so that its source-depth reads fall into few lines while each query's FL
-  // outputs stay contiguous.  A block step writes R S consecutive pairs.
-  const int FLP = FL / P;
-  const int fi = i % FLP;
-  const int qi = (i / FLP) % R;
-  const int s0 = (i / (FLP * R)) * FL + fi * P;
-  int q = qb + qi;
   if (q >= q_end) return;
   int t = q / hw;
   int iy = (q - t * hw) / a.w;
@@ -220,7 +240,6 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   const float wf = (float)a.w, hf = (float)a.h;
   Idx o = (Idx)q * (Idx)S + (Idx)s0;
   const Idx o_step = (Idx)R * (Idx)S;
-  float z = a.depth[q];
   for (; q < q_end; q += R, o += o_step) {
     const float zn = q + R < q_end ? a.depth[q + R] : 0.f;  // next query's depth, in flight meanwhile
     const float u0 = (float)jx;
