@@ -272,7 +272,9 @@ crc_status crc_gather(const crc_shape* shape, const void* pool, int32_t num_slab
  *   d_uv     device [N_q][S][2] fp32 u^ (NaN where undefined), S = k*F.
  *   d_cell   device [N_q][S] int32: y*w + x, or -1 when not valid.  May be NULL.
  *   d_valid  device [N_q][S] uint8: 1 valid, 0 not.
- * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_CUDA.
+ * Errors: CRC_ERR_INVALID_ARG; CRC_ERR_UNSUPPORTED when d_uv is not 8-byte aligned
+ * or when the bank's depth array (capacity * F * h * w values) exceeds 2^31 - 1
+ * values; CRC_ERR_CUDA.
  */
 crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const float* d_depth, const crc_bank* bank,
                           const int32_t* d_idx, const int32_t* d_count, int32_t k, float eps, float* d_uv,

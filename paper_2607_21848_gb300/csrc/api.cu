@@ -315,6 +315,8 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
   if (k < 1 || k > CRC_MAX_K || isnan(eps) || eps < 0.f) return CRC_ERR_INVALID_ARG;
   if (!frames_ok(cur, shape->F)) return CRC_ERR_INVALID_ARG;
   if (((uintptr_t)d_uv & 7u) != 0) return CRC_ERR_UNSUPPORTED;
+  // the kernel addresses the bank's depth array with 32-bit offsets
+  if ((int64_t)bank->capacity * shape->F * shape->h * shape->w > INT32_MAX) return CRC_ERR_UNSUPPORTED;
   crc::CorrespondArgs a;
   memset(&a, 0, sizeof(a));
   pack_frames(a.cur, cur, shape->F);

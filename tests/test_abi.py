@@ -95,3 +95,21 @@ def test_ctypes_layout_matches_header():
     }
     for k, v in ct.items():
         assert int(got[k]) == v, (k, got[k], v)
+
+
+def test_correspond_rejects_a_bank_beyond_32_bit_depth_offsets(lib):
+    """A bank whose depth array holds 2^31 or more values is rejected on the host,
+    before any CUDA call: the reprojection kernel addresses it with 32-bit offsets.
+    The device pointers are placeholders that nothing dereferences."""
+    F, h, w = 3, 45, 80
+    cap = (2**31) // (F * h * w) + 1
+    shape = _abi.crc_shape(1, 1, 64, F, h, w, _abi.CRC_F32)
+    fake = 1 << 20
+    bank = _abi.crc_bank(cap, 1, fake, fake, fake, fake, fake)
+    frames = (_abi.crc_frame * F)()
+    for f in range(F):
+        frames[f].K[:] = [40.0, 0.0, 39.5, 0.0, 40.0, 22.0, 0.0, 0.0, 1.0]
+        frames[f].R[:] = [1.0, 0.0, 0.0, 0.0, 1.0, 0.0, 0.0, 0.0, 1.0]
+    args = (C.byref(shape), frames, fake, C.byref(bank), fake, None, 1, 0.05, fake, None, fake, None)
+    assert cap * F * h * w > 2**31 - 1 >= (cap - 1) * F * h * w  # one chunk past the limit
+    assert lib.crc_correspond(*args) == _abi.CRC_ERR_UNSUPPORTED
