@@ -215,7 +215,7 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
  * crc_retrieve — Sec. 4.2, Eq. 1 over bank chunks j in [0, bank_count):
  *   s(j) = ||c_j - c_n||_2 / E + w_v (1 - v_j . v_n)
  *   A_n  = { j : ||c_j - c_n||/E <= tau_c, v_j . v_n >= cos_tau_v, n - j >= delta }
- * where (c_n, v_n) summarise `cur` (host [F] frames of current chunk n) exactly as
+ * where (c_n, v_n) summarise `cur` (host [F] frames of current chunk n >= 0) exactly as
  * crc_bank_insert_poses does.  Scores are fp64 without FMA contraction, in the
  * order dx*dx+dy*dy+dz*dz, sqrt, /E; dot product left to right.
  *

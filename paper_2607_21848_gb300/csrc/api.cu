@@ -259,7 +259,7 @@ crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shap
   if (st) return st;
   if ((st = check_bank(bank, cache != nullptr))) return st;
   if (!cur || !p || !d_idx || !d_count) return CRC_ERR_INVALID_ARG;
-  if (bank_count < 0 || bank_count > bank->capacity) return CRC_ERR_INVALID_ARG;
+  if (bank_count < 0 || bank_count > bank->capacity || n < 0) return CRC_ERR_INVALID_ARG;
   if (p->k < 1 || p->k > CRC_MAX_K || !(p->E > 0.0) || isnan(p->w_v) || isnan(p->tau_c) || isnan(p->cos_tau_v))
     return CRC_ERR_INVALID_ARG;
   if (!frames_ok(cur, shape->F)) return CRC_ERR_INVALID_ARG;

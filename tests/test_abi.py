@@ -113,3 +113,20 @@ def test_correspond_rejects_a_bank_beyond_32_bit_depth_offsets(lib):
     args = (C.byref(shape), frames, fake, C.byref(bank), fake, None, 1, 0.05, fake, None, fake, None)
     assert cap * F * h * w > 2**31 - 1 >= (cap - 1) * F * h * w  # one chunk past the limit
     assert lib.crc_correspond(*args) == _abi.CRC_ERR_UNSUPPORTED
+
+
+def test_retrieve_rejects_a_negative_chunk_index(lib):
+    """The temporal gate n - j >= delta is evaluated in 32-bit integers; n is the
+    index of the current chunk and must not be negative.  Rejected on the host,
+    before any CUDA call; the device pointers are placeholders."""
+    F, h, w = 3, 8, 8
+    shape = _abi.crc_shape(1, 1, 64, F, h, w, _abi.CRC_F32)
+    fake = 1 << 20
+    bank = _abi.crc_bank(4, 1, fake, fake, fake, fake, fake)
+    frames = (_abi.crc_frame * F)()
+    for f in range(F):
+        frames[f].K[:] = [4.0, 0.0, 3.5, 0.0, 4.0, 3.5, 0.0, 0.0, 1.0]
+        frames[f].R[:] = [1.0, 0.0, 0.0, 0.0, 1.0, 0.0, 0.0, 0.0, 1.0]
+    params = _abi.crc_retrieval(1.0, 0.5, float("inf"), -1.0, 1, 1, -1, 0, 0)
+    assert lib.crc_retrieve(C.byref(bank), 4, C.byref(shape), frames, -1, C.byref(params), None, None, fake, None,
+                            fake, None) == _abi.CRC_ERR_INVALID_ARG
