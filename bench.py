@@ -236,7 +236,7 @@ E2E_BUFFERS = 3
 
 
 def run_e2e(W, stream, steps: int):
-    """The step through the public API with host buffers, pipelined on two copy streams.
+    """The step through the public API with host buffers, pipelined against one copy stream.
 
     Every step copies its inputs (Q, the new chunk's K/V, its depth) from pinned host
     memory and copies O back, on one copy stream: the step's copies fit in its kernel
