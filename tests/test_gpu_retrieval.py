@@ -11,7 +11,7 @@ import torch
 
 import oracle
 import synth
-from paper_2607_21848_gb300 import api
+from paper_2607_21848_gb300 import _abi, api
 from tests import _gpu
 
 pytestmark = pytest.mark.gpu
@@ -58,7 +58,7 @@ def test_retrieve_topk_bit_exact(cfg):
     wl = synth.make_workload(cfg)
     bank, shp = _gpu.make_bank(wl, _gpu.dev_dtype(wl))
     _gpu.insert_poses(bank, shp, wl.bank_frames)
-    for k in sorted({wl.k, 1, 5}):
+    for k in sorted({wl.k, 1, 5, _abi.CRC_MAX_K}):
         oi, os_, oc, _ = _gpu.oracle_retrieve(wl, k=k)
         gi, gs, gc = _gpu_retrieve(wl, bank, shp, wl.bank_size, wl.n, wl.cur_frames, k)
         assert gc == oc
