@@ -45,8 +45,20 @@ def _peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         d = json.load(open(p))
-        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"], src="measured")
-    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"], src="measured",
+                    sus_mhz=d.get("clocks_under_load", {}).get("sm_mhz_median"))
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback", sus_mhz=None)
+
+
+# One tcgen05.mma of M = N = 128, K = 16 (bf16 in, fp32 accumulate: 2 * 128 * 128 * 16 FLOP)
+# occupies an SM's tensor core for 64 clocks on this GPU (measured with single-instruction
+# timing loops), so the dense issue ceiling is 8192 FLOP per SM clock.
+MMA_FLOP_PER_SM_CLOCK = 2 * 128 * 128 * 16 / 64
+
+
+def issue_ceiling_tflops(sm_mhz, sms: int = 152):
+    """Dense bf16 tensor-core ceiling at the sampled SM clock (context beside the measured peak)."""
+    return None if not sm_mhz else MMA_FLOP_PER_SM_CLOCK * sms * sm_mhz * 1e6 / 1e12
 
 
 # ---------------------------------------------------------------------------- clocks
@@ -508,7 +520,7 @@ def stream_context(device, seed: int):
 
     wl = synth.make_workload(5)
     cfg = crs.StreamConfig(L=wl.L, H=wl.H, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2,
-                           capacity=wl.bank_size, num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c,
+                           capacity=wl.bank_size, num_slabs=wl.bank_size, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c,
                            cos_tau_v=wl.cos_tau_v, delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps)
     st = crs.ChunkStream(cfg, device=device)
     Nc = cfg.Nc
@@ -735,7 +747,7 @@ def main():
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
     sweep = shapes = modes = stream_ctx = None
     if not args.no_context:
-        from paper_2607_21848_gb300.sweeps import correspond_sweep
+        from sweeps import correspond_sweep
 
         sweep = correspond_sweep(device)
         sweep["iid_depth"] = {key: val for key, val in correspond_sweep(device, depth="iid").items()
@@ -746,6 +758,20 @@ def main():
 
     peaks = _peaks()
     attn_tflops = alg["flops"] / stage["attention"] / 1e12
+    clk_summary = clk.summary()
+    hbm_rooflines = {
+        "peak": peaks["hbm"], "unit": "GB/s", "peak_source": f"{peaks['src']} HBM copy",
+        "retrieve_gather": {"kernel": "retrieve_gather_kernel", "gbs": alg["gather_bytes"] / stage["retrieve"] / 1e9,
+                            "bytes": alg["gather_bytes"]},
+        "cache_update": {"kernel": "cache_update_kernel", "gbs": alg["update_bytes"] / stage["update"] / 1e9,
+                         "bytes": alg["update_bytes"]},
+    }
+    if sweep is not None:
+        hbm_rooflines["correspond_sweep"] = {"kernel": "correspond_kernel", "gbs": sweep["gbs"], "bytes": sweep["bytes"],
+                                             "what": "126 MB reprojection sweep (4 x 180 x 320 queries, 32 frames)"}
+    for key in ("retrieve_gather", "cache_update", "correspond_sweep"):
+        if key in hbm_rooflines:
+            hbm_rooflines[key]["frac"] = hbm_rooflines[key]["gbs"] / peaks["hbm"]
     line = {
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
@@ -757,18 +783,27 @@ def main():
             "correspond_ms": stage["correspond"] * 1e3,
             "correspond_gbs": alg["reproj_bytes"] / stage["correspond"] / 1e9,
             "attention_ms": stage["attention"] * 1e3, "attention_tflops": attn_tflops,
-            "attention_frac_of_bf16_peak": attn_tflops / peaks["bf16_sus"],
+            "attention_frac_of_bf16_peak": attn_tflops / peaks["bf16"],
             "retrieve_frac_of_hbm_peak": alg["gather_bytes"] / stage["retrieve"] / 1e9 / peaks["hbm"],
             "note": "medians of the timed steps; min_ms the fastest step of each stage",
             "min_ms": {nm: t * 1e3 for nm, t in stage_min.items()},
         },
         "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel", "achieved": attn_tflops,
-                     "peak": peaks["bf16_sus"], "unit": "TFLOP/s", "frac": attn_tflops / peaks["bf16_sus"],
-                     "peak_source": f"{peaks['src']} bf16 sustained (kernel timed inside a long step)",
-                     "frac_of_burst": attn_tflops / peaks["bf16"],
+                     "peak": peaks["bf16"], "unit": "TFLOP/s", "frac": attn_tflops / peaks["bf16"],
+                     "peak_source": (f"{peaks['src']} bf16 burst (cuBLAS); the attention call is timed inside a "
+                                     f"{step_s * args.steps:.2f} s loop at the clock in `clocks`"),
+                     "frac_of_sustained": attn_tflops / peaks["bf16_sus"],
+                     "sustained_note": (f"the sustained figure was taken over a seconds-long GEMM loop at a median "
+                                        f"{peaks['sus_mhz']} MHz; context only"),
+                     "issue_ceiling": issue_ceiling_tflops(clk_summary["sm_mhz"]),
+                     "frac_of_issue_ceiling": (attn_tflops / issue_ceiling_tflops(clk_summary["sm_mhz"])
+                                               if clk_summary["sm_mhz"] else None),
+                     "issue_ceiling_note": "152 SMs x 8192 FLOP per clock (one 128x128x16 MMA per 64 clocks) x "
+                                           "the median SM clock sampled in the timed region",
                      "traffic": (ATTN_DRAM_BYTES_PER_LAYER[(wl.H, wl.Nq, wl.n_keys)] * wl.L
                                  if (wl.H, wl.Nq, wl.n_keys) in ATTN_DRAM_BYTES_PER_LAYER else None),
-                     "traffic_algorithmic": alg["attn_bytes"]},
+                     "traffic_algorithmic": alg["attn_bytes"],
+                     "hbm": hbm_rooflines},
         "e2e": {"value": whole_job_tflops(alg["flops"], e2e_s, world), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
                 "pipelining": f"{E2E_BUFFERS} device buffer sets; on one copy stream, uploads run up to "
@@ -779,7 +814,7 @@ def main():
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
                   "note": "one step captured in a CUDA graph and replayed"},
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,
-        "clocks": clk.summary(),
+        "clocks": clk_summary,
     }
     if context is not None:
         line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path",
@@ -789,7 +824,7 @@ def main():
             sweep["frac_of_hbm_peak"] = sweep["gbs"] / peaks["hbm"]
             sweep["iid_depth"]["frac_of_hbm_peak"] = sweep["iid_depth"]["gbs"] / peaks["hbm"]
         for v in (shapes or {}).values():
-            v["frac_of_bf16_peak"] = v["tflops"] / peaks["bf16_sus"]
+            v["frac_of_bf16_peak"] = v["tflops"] / peaks["bf16"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cb = oracle_sample(args.config, args.layers, 10.0)
         line["cpu_baseline"] = {

@@ -111,14 +111,23 @@ typedef struct {
   crc_segment seg[CRC_MAX_SEGMENTS];
 } crc_cache;
 
-/* Memory bank of every chunk generated so far (Sec. 4.2: evicted chunks stay
- * retrievable).  Device arrays, caller-allocated:
+/* Memory bank of the chunks generated so far (Sec. 4.2: chunks evicted from the
+ * recent window stay retrievable).  Device arrays, caller-allocated:
  *   frames [capacity][F][21]  fp64 crc_frame records of every chunk
  *   centre [capacity][3]      fp64 chunk centre c_j (written by the library)
  *   view   [capacity][3]      fp64 unit view direction v_j (written by the library)
  *   depth  [capacity][F][h][w] fp32 planar metric depth of every chunk
  *   kv     [num_slabs][2][L][N_c][H][d] K (index 0) and V (index 1) slabs, dense,
- *          dtype of the call; chunk j lives in slab j % num_slabs. */
+ *          dtype of the call; chunk j lives in slab j % num_slabs.
+ *   slab_chunk [num_slabs] int32, or NULL: the chunk whose K/V slab s holds (-1 for
+ *          none; the caller fills it with -1 before the first update).  When it is
+ *          given, crc_cache_update records every chunk it writes, and retrieval only
+ *          admits chunks whose slab still holds them: with num_slabs < capacity a
+ *          chunk stops being retrievable once chunk j + num_slabs overwrites its slab.
+ *          When it is NULL the caller guarantees that slab j % num_slabs holds chunk
+ *          j's K/V for every chunk that can be retrieved (e.g. num_slabs >= the
+ *          number of chunks, or a pool of synthetic slabs).
+ * Poses, pose summaries and depth are kept for all `capacity` chunks. */
 typedef struct {
   int32_t capacity;
   int32_t num_slabs;
@@ -127,6 +136,7 @@ typedef struct {
   double* view;
   float* depth;
   void* kv;
+  int32_t* slab_chunk;
 } crc_bank;
 
 /* Eq. 1 parameters and the empty-set fallback of Sec. 4.2. */
@@ -199,9 +209,10 @@ crc_status crc_bank_insert_poses(const crc_bank* bank, const crc_shape* shape, i
  *                centre and view direction (as crc_bank_insert_poses).
  *   d_depth      device [F][h][w] fp32 depth; copied to bank->depth[chunk].
  *   d_k, d_v     device [L][N_c][H][d] dense, dtype of the call; copied to slab
- *                chunk % num_slabs of bank->kv and, if window_offset >= 0, to
- *                cache keys [window_offset, window_offset + N_c) of every layer.
- *                Both may be NULL (poses and depth only).
+ *                chunk % num_slabs of bank->kv (and bank->slab_chunk[chunk %
+ *                num_slabs] = chunk when the bank tracks its slabs) and, if
+ *                window_offset >= 0, to cache keys [window_offset, window_offset + N_c)
+ *                of every layer.  Both may be NULL (poses and depth only).
  *   cache        may be NULL when window_offset < 0.
  * The sink and the other cache keys are not touched.
  * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE (window slot outside the cache),
@@ -215,6 +226,8 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
  * crc_retrieve — Sec. 4.2, Eq. 1 over bank chunks j in [0, bank_count):
  *   s(j) = ||c_j - c_n||_2 / E + w_v (1 - v_j . v_n)
  *   A_n  = { j : ||c_j - c_n||/E <= tau_c, v_j . v_n >= cos_tau_v, n - j >= delta }
+ * restricted, when bank->slab_chunk is given, to chunks whose K/V slab still holds
+ * them (a window-extension chunk whose slab was overwritten leaves its slot empty)
  * where (c_n, v_n) summarise `cur` (host [F] frames of current chunk n >= 0) exactly as
  * crc_bank_insert_poses does.  Scores are fp64 without FMA contraction, in the
  * order dx*dx+dy*dy+dz*dz, sqrt, /E; dot product left to right.
@@ -229,11 +242,27 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
  * d_idx[r] >= 0, keys [offset, offset+N_c) of every layer receive the K and V
  * of slab d_idx[r] % num_slabs (the gather), the keys re-positioned by `rope`
  * when it is not NULL.  Everything stays on the device.
- * Errors: CRC_ERR_INVALID_ARG, CRC_ERR_SHAPE, CRC_ERR_UNSUPPORTED, CRC_ERR_CUDA.
+ *
+ * Every bank entry is scored once.  Banks of more than 512 entries are split over
+ * several blocks whose candidates meet in `d_workspace`: device memory of at least
+ * crc_retrieve_workspace_size(bank_count, k) bytes, 16-byte aligned, owned by the
+ * caller and written by the call (its previous contents do not matter).  When that
+ * size is 0 the workspace may be NULL.  One workspace serves one call at a time:
+ * calls that may overlap on the GPU need workspaces of their own.
+ * Enqueued work: a 4-byte memset of the workspace (when it is used), the scoring
+ * launch and, with a cache, the gather launch.
+ * Errors: CRC_ERR_INVALID_ARG (also a missing, short or misaligned workspace, a
+ * non-finite E or w_v), CRC_ERR_SHAPE, CRC_ERR_UNSUPPORTED, CRC_ERR_CUDA.
  */
 crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
                         int32_t n, const crc_retrieval* p, const crc_cache* cache, const crc_rope* rope,
-                        int32_t* d_idx, double* d_score, int32_t* d_count, cudaStream_t s);
+                        int32_t* d_idx, double* d_score, int32_t* d_count, void* d_workspace,
+                        size_t workspace_bytes, cudaStream_t s);
+
+/* Workspace bytes crc_retrieve needs for a bank of `bank_count` entries and k
+ * slots: 0 up to 512 entries, else 16 bytes per (block of 512 entries, slot) plus
+ * 256, rounded up (under 300 KB for any bank).  0 for invalid arguments. */
+size_t crc_retrieve_workspace_size(int32_t bank_count, int32_t k);
 
 /*
  * crc_gather — the gather half of crc_retrieve for a second cache that mirrors
@@ -289,6 +318,9 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
                                 on the tensor-core kernel, which adds the bonus to each biased tile's
                                 scores in the softmax; otherwise the SIMT kernel.  Not combined with
                                 CRC_ATTN_SKIP_FAR, which is then ignored. */
+#define CRC_ATTN_BIAS_DIRECT 8  /* tensor-core kernel, Eq. 2 form: evaluate the bias per score in the
+                                   softmax (exact to fp32 rounding) even where the tensor-core
+                                   expansion is within its error limit (see crc_biased_attention) */
 #define CRC_ATTN_SKIP_FAR 4  /* opt-in approximation (tensor-core kernel, Eq. 2 form): a KV tile of a
                                 retrieved frame is skipped for a block of 256 queries when every one of
                                 them has a valid correspondence in that frame and the distance from the
@@ -317,17 +349,89 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
  *             an internal pipeline barrier (the output is then not valid).
  * bf16 (d = 128) runs on the tcgen05 tensor-core kernel with fp32 softmax and
  * accumulation, in either bias form; fp32 or CRC_ATTN_SIMT run the SIMT kernel in fp32.
+ * Eq. 2 on the tensor-core kernel: the bias is added to S by the tensor core itself, as
+ * a K = 16 extension of q.k (a rank-4 expansion of ||u_k - u^||^2 about the frame centre).
+ * Its terms cancel near the correspondence, so its error grows with the grid: at most
+ * crc_bias_expansion_bound(lambda, sigma, h, w) = 2^-23 C (w^2 + h^2) in base-2 logit
+ * units, C = lambda log2(e) / (2 sigma^2).  Where that exceeds 2^-9 (the bf16 rounding
+ * of the softmax weights; e.g. lambda / sigma^2 > 2.69 on a 45 x 80 grid, > 6.3 on
+ * 30 x 52) the kernel adds the bias per score in the softmax instead, exact to fp32
+ * rounding, at a lower throughput; CRC_ATTN_BIAS_DIRECT selects that everywhere.
  * The tensor-core kernel takes at most 640 KV tiles of 128 keys per call (each
  * segment is cut into tiles from its start, a retrieved segment per frame: up to
  * 81 920 keys) and h*w <= 65535; beyond that the call returns CRC_ERR_UNSUPPORTED
  * before any launch, and CRC_ATTN_SIMT takes it.
  * Errors: CRC_ERR_INVALID_ARG (also unknown flag bits), CRC_ERR_SHAPE,
- * CRC_ERR_UNSUPPORTED (dtype, d, alignment, device without sm_103a), CRC_ERR_CUDA.
+ * CRC_ERR_UNSUPPORTED (dtype, d, alignment -- d_uv must be 8-byte aligned --, device
+ * without sm_103a), CRC_ERR_CUDA.
  */
 crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_cache* cache, crc_tensor o,
                                 float* d_lse, int32_t n_q, const float* d_uv, const uint8_t* d_valid, int32_t k,
                                 const int32_t* d_slot_chunk, float lambda, float sigma, int32_t flags,
                                 int32_t* d_status, cudaStream_t s);
+
+/* ---- a whole chunk step from a device-resident descriptor --------------------
+ *
+ * A chunk step of a stream (Sec. 4.2 "Cache layout" and "Loop-closure retrieval": one
+ * step per generated chunk) is crc_cache_update, crc_retrieve, crc_correspond and
+ * crc_biased_attention with values that change from step to step: the chunk index,
+ * the window slot that receives the chunk, the fallback chunk, the re-positioning
+ * target, which window segments hold a chunk yet, and the chunk's camera frames.
+ * crc_chunk_step reads those from a descriptor in device memory, so that one captured
+ * sequence of its launches (a CUDA graph) serves every step of the stream: the caller
+ * rewrites the descriptor (for instance with a host-to-device copy captured in the
+ * same graph, from a pinned buffer it rewrites before each replay) and replays. */
+
+/* The per-step values, in device memory (8-byte aligned). */
+typedef struct {
+  int32_t n;               /* current chunk; the bank holds chunks 0..n (n < bank capacity)     */
+  int32_t window_offset;   /* first cache key of the slot that receives chunk n (-1: none)      */
+  int32_t ext_first;       /* crc_retrieval.ext_first of this step                              */
+  int32_t rope_pos_slot0;  /* crc_rope.pos_slot0 of this step (unused without re-positioning)   */
+  int32_t seg_length[CRC_MAX_SEGMENTS]; /* each cache segment's length this step, 0 ..
+                                           its length in the plan (a retrieved one: 0 or N_c) */
+  crc_frame frames[CRC_MAX_FRAMES];     /* the current chunk's frames (first F used)           */
+} crc_step;
+
+/* What stays fixed over the steps: every pointer is captured by the launches. */
+typedef struct {
+  crc_shape shape;
+  crc_bank bank;             /* with its K/V slab pool                                        */
+  crc_cache cache;           /* segment offsets, kinds, slots; lengths are the largest ones    */
+  crc_retrieval retrieval;   /* ext_first is taken from the descriptor                        */
+  crc_rope rope;             /* pairs = 0: no re-positioning; pos_slot0 from the descriptor    */
+  float eps;                 /* Eq. 4 tolerance (INFINITY: off)                                */
+  float lambda, sigma;       /* Eq. 2                                                          */
+  int32_t attn_flags;        /* CRC_ATTN_* as for crc_biased_attention                         */
+  /* per-step inputs, device, rewritten by the caller before each step */
+  const float* d_depth;      /* [F][h][w] depth of chunk n                                     */
+  const void* d_k;           /* [L][N_c][H][d] K and V of chunk n (dense)                       */
+  const void* d_v;
+  crc_tensor q;              /* [L][N_c][H][d] queries                                         */
+  /* outputs, device */
+  crc_tensor o;
+  float* d_lse;              /* [L][H][N_c] or NULL                                            */
+  int32_t* d_idx;            /* [k]                                                            */
+  double* d_score;           /* [k] or NULL                                                    */
+  int32_t* d_count;          /* [1]                                                            */
+  float* d_uv;               /* [N_c][k F][2], 8-byte aligned                                   */
+  int32_t* d_cell;           /* [N_c][k F] or NULL                                             */
+  uint8_t* d_valid;          /* [N_c][k F]                                                     */
+  int32_t* d_status;         /* [1], required: CRC_STEP_BAD_DESCRIPTOR when a kernel finds the
+                                descriptor out of range (it then writes nothing else), or a
+                                pipeline timeout code of the attention kernel                   */
+  void* d_workspace;         /* crc_retrieve_workspace_size(bank.capacity, k) bytes            */
+  size_t workspace_bytes;
+} crc_step_plan;
+
+#define CRC_STEP_BAD_DESCRIPTOR 100
+
+
+/* Bound on the error of the tensor-core expansion of the Eq. 2 bias on an h x w grid,
+ * in base-2 logit units: 2^-23 lambda log2(e) / (2 sigma^2) (w^2 + h^2); +inf where
+ * the key coordinates are not exact in bf16 (w or h above 256, or
+ * (w-1)^2 + (h-1)^2 >= 2^16), which always takes the per-score form.  Host only. */
+double crc_bias_expansion_bound(float lambda, float sigma, int32_t h, int32_t w);
 
 #ifdef __cplusplus
 }

@@ -86,10 +86,14 @@ def retrieval_terms(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n
 
 def retrieve(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n: np.ndarray, n: int,
              E: float, w_v: float, tau_c: float, cos_tau_v: float, delta: int, k: int,
-             exclude_sink: bool = False):
+             exclude_sink: bool = False, resident: Optional[np.ndarray] = None):
     """Eq. 1: score every historical chunk j, keep the admissible set A_n, and return
     the k admissible chunks closest in pose (ascending (s, j)).  With exclude_sink
     the anchor chunk j = 0 (always in the cache already) is never admissible.
+
+    resident [B] bool (optional): chunks whose keys and values are still held.  The
+    paper keeps every chunk re-encodable (Sec. 4.2); a store of bounded size can
+    only reinstate the chunks it still holds, so the others are not admissible.
 
     Returns (idx [k] int32 padded with -1, score [k] fp64 padded with +inf, count).
     """
@@ -99,6 +103,8 @@ def retrieve(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n: np.nd
     adm = (dist <= tau_c) & (dot >= cos_tau_v) & ((n - j) >= delta)
     if exclude_sink:
         adm &= j != 0
+    if resident is not None:
+        adm &= np.asarray(resident, dtype=bool)[:B]
     cand = sorted((float(s[i]), int(i)) for i in np.nonzero(adm)[0])
     count = min(k, len(cand))
     idx = np.full(k, -1, dtype=np.int32)
@@ -108,15 +114,20 @@ def retrieve(bank_c: np.ndarray, bank_v: np.ndarray, c_n: np.ndarray, v_n: np.nd
     return idx, score, count
 
 
-def fill_slots(idx: np.ndarray, count: int, ext_first: int, ext_min: int) -> np.ndarray:
+def fill_slots(idx: np.ndarray, count: int, ext_first: int, ext_min: int,
+               resident: Optional[np.ndarray] = None) -> np.ndarray:
     """Chunk held by each retrieved slot.  Slots r < count hold the retrieval result;
     the rest extend the recent window with the next-older chunks ext_first,
-    ext_first-1, ... while they are >= ext_min, else stay empty (-1)."""
+    ext_first-1, ... while they are >= ext_min (and, given `resident`, still held),
+    else stay empty (-1)."""
     k = idx.shape[0]
     out = np.array(idx, dtype=np.int32)
     for r in range(count, k):
         e = ext_first - (r - count)
-        out[r] = e if (ext_first >= 0 and e >= ext_min) else -1
+        ok = ext_first >= 0 and e >= ext_min
+        if ok and resident is not None:
+            ok = bool(resident[e])
+        out[r] = e if ok else -1
     return out
 
 

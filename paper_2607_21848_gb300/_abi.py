@@ -34,6 +34,7 @@ CRC_ATTN_DEFAULT = 0
 CRC_ATTN_SIMT = 1
 CRC_ATTN_GAUSSIAN = 2
 CRC_ATTN_SKIP_FAR = 4
+CRC_ATTN_BIAS_DIRECT = 8
 
 
 class crc_frame(C.Structure):
@@ -61,7 +62,7 @@ class crc_cache(C.Structure):
 
 class crc_bank(C.Structure):
     _fields_ = [("capacity", C.c_int32), ("num_slabs", C.c_int32), ("frames", C.c_void_p), ("centre", C.c_void_p),
-                ("view", C.c_void_p), ("depth", C.c_void_p), ("kv", C.c_void_p)]
+                ("view", C.c_void_p), ("depth", C.c_void_p), ("kv", C.c_void_p), ("slab_chunk", C.c_void_p)]
 
 
 class crc_retrieval(C.Structure):
@@ -86,7 +87,8 @@ _SIGS = {
                                      C.c_void_p, _P(crc_cache), C.c_int32, C.c_void_p]),
     "crc_retrieve": (C.c_int32, [_P(crc_bank), C.c_int32, _P(crc_shape), _P(crc_frame), C.c_int32,
                                  _P(crc_retrieval), _P(crc_cache), _P(crc_rope), C.c_void_p, C.c_void_p, C.c_void_p,
-                                 C.c_void_p]),
+                                 C.c_void_p, C.c_size_t, C.c_void_p]),
+    "crc_retrieve_workspace_size": (C.c_size_t, [C.c_int32, C.c_int32]),
     "crc_gather": (C.c_int32, [_P(crc_shape), C.c_void_p, C.c_int32, C.c_void_p, C.c_int32, _P(crc_cache),
                                _P(crc_rope), C.c_void_p]),
     "crc_correspond": (C.c_int32, [_P(crc_shape), _P(crc_frame), C.c_void_p, _P(crc_bank), C.c_void_p, C.c_void_p,
@@ -94,6 +96,7 @@ _SIGS = {
     "crc_biased_attention": (C.c_int32, [_P(crc_shape), crc_tensor, _P(crc_cache), crc_tensor, C.c_void_p, C.c_int32,
                                          C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_float, C.c_float,
                                          C.c_int32, C.c_void_p, C.c_void_p]),
+    "crc_bias_expansion_bound": (C.c_double, [C.c_float, C.c_float, C.c_int32, C.c_int32]),
 }
 
 EXPORTED = tuple(_SIGS)

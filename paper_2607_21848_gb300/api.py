@@ -25,6 +25,7 @@ ATTN_DEFAULT = _abi.CRC_ATTN_DEFAULT
 ATTN_SIMT = _abi.CRC_ATTN_SIMT
 ATTN_GAUSSIAN = _abi.CRC_ATTN_GAUSSIAN
 ATTN_SKIP_FAR = _abi.CRC_ATTN_SKIP_FAR
+ATTN_BIAS_DIRECT = _abi.CRC_ATTN_BIAS_DIRECT
 
 
 def _dtype_code(dt: torch.dtype) -> int:
@@ -67,11 +68,19 @@ def tensor_view(t: torch.Tensor) -> _abi.crc_tensor:
     return _abi.crc_tensor(_ptr(t), t.stride(0), t.stride(1), t.stride(2))
 
 
+def crc_retrieve_workspace_size(bank_count: int, k: int) -> int:
+    return int(_abi.load().crc_retrieve_workspace_size(bank_count, k))
+
+
 class Bank:
-    """Device memory of the chunk bank (frames, pose summaries, depth, K/V slabs)."""
+    """Device memory of the chunk bank (frames, pose summaries, depth, K/V slabs).
+
+    track_slabs: keep the chunk held by each K/V slab (crc_bank.slab_chunk), so that
+    retrieval never returns a chunk whose slab a newer chunk has overwritten.  The
+    bank also owns the retrieval workspace for its capacity (crc_retrieve)."""
 
     def __init__(self, capacity: int, F: int, h: int, w: int, L: int, H: int, d: int, dtype: torch.dtype,
-                 num_slabs: int, device="cuda", with_kv: bool = True):
+                 num_slabs: int, device="cuda", with_kv: bool = True, track_slabs: bool = False):
         self.capacity, self.F, self.h, self.w = capacity, F, h, w
         self.L, self.H, self.d, self.dtype, self.num_slabs = L, H, d, dtype, num_slabs
         self.frames = torch.zeros(capacity, F, 21, dtype=torch.float64, device=device)
@@ -80,10 +89,15 @@ class Bank:
         self.depth = torch.zeros(capacity, F, h, w, dtype=torch.float32, device=device)
         self.kv = (torch.zeros(num_slabs, 2, L, F * h * w, H, d, dtype=dtype, device=device)
                    if with_kv else None)
+        self.slab_chunk = (torch.full((num_slabs,), -1, dtype=torch.int32, device=device)
+                           if track_slabs and with_kv else None)
+        ws = crc_retrieve_workspace_size(capacity, _abi.CRC_MAX_K)
+        self.workspace = torch.empty(max(ws, 16), dtype=torch.uint8, device=device) if ws else None
 
     def struct(self) -> _abi.crc_bank:
         return _abi.crc_bank(self.capacity, self.num_slabs, _ptr(self.frames), _ptr(self.centre), _ptr(self.view),
-                             _ptr(self.depth), _ptr(self.kv) if self.kv is not None else None)
+                             _ptr(self.depth), _ptr(self.kv) if self.kv is not None else None,
+                             _ptr(self.slab_chunk))
 
 
 class Cache:
@@ -127,6 +141,10 @@ def rope_params(channel0: int, pairs: int, theta: float, interleaved: bool, pos_
     return _abi.crc_rope(channel0, pairs, int(bool(interleaved)), pos_slot0, pos_stride, frame_pos0, float(theta))
 
 
+def crc_bias_expansion_bound(lam: float, sigma: float, h: int, w: int) -> float:
+    return float(_abi.load().crc_bias_expansion_bound(lam, sigma, h, w))
+
+
 def crc_version() -> str:
     return _abi.load().crc_version().decode()
 
@@ -154,15 +172,19 @@ def crc_cache_update(bank: Bank, shp: _abi.crc_shape, chunk: int, frames: np.nda
 
 def crc_retrieve(bank: Bank, bank_count: int, shp: _abi.crc_shape, cur_frames: np.ndarray, n: int,
                  params: _abi.crc_retrieval, cache: Optional[Cache], idx: torch.Tensor, score: Optional[torch.Tensor],
-                 count: torch.Tensor, stream=None, rope: Optional[_abi.crc_rope] = None) -> None:
+                 count: torch.Tensor, stream=None, rope: Optional[_abi.crc_rope] = None,
+                 workspace: Optional[torch.Tensor] = None) -> None:
+    """`workspace` defaults to the bank's own (sized for its capacity)."""
     lib = _abi.load()
     fr = frames_struct(cur_frames)
     b = bank.struct()
     cs = cache.struct() if cache is not None else None
+    ws = bank.workspace if workspace is None else workspace
     _abi.check("crc_retrieve",
                lib.crc_retrieve(C.byref(b), bank_count, C.byref(shp), fr, n, C.byref(params),
                                 C.byref(cs) if cs is not None else None, C.byref(rope) if rope is not None else None,
-                                _ptr(idx), _ptr(score), _ptr(count), _stream(stream)))
+                                _ptr(idx), _ptr(score), _ptr(count), _ptr(ws),
+                                0 if ws is None else ws.numel() * ws.element_size(), _stream(stream)))
 
 
 def crc_gather(shp: _abi.crc_shape, pool: torch.Tensor, idx: torch.Tensor, k: int, cache: Cache,

@@ -59,7 +59,7 @@ bool frames_ok(const crc_frame* fr, int F) {
 
 crc_status check_bank(const crc_bank* b, bool need_kv) {
   if (!b || b->capacity < 1 || !b->frames || !b->centre || !b->view || !b->depth) return CRC_ERR_INVALID_ARG;
-  if (need_kv && (!b->kv || b->num_slabs < 1)) return CRC_ERR_INVALID_ARG;
+  if ((need_kv || b->slab_chunk) && (!b->kv || b->num_slabs < 1)) return CRC_ERR_INVALID_ARG;
   return CRC_OK;
 }
 
@@ -238,6 +238,7 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
     a.v_src = static_cast<const char*>(d_v);
     const int64_t slab_bytes = 2LL * shape->L * nc * row_bytes;
     a.slab = static_cast<char*>(bank->kv) + (int64_t)(chunk % bank->num_slabs) * slab_bytes;
+    a.slab_owner = bank->slab_chunk ? bank->slab_chunk + chunk % bank->num_slabs : nullptr;
     if (window_offset >= 0) {
       if ((st = check_cache(cache, shape))) return st;
       if ((int64_t)window_offset + nc > cache->n_keys) return CRC_ERR_SHAPE;
@@ -251,23 +252,38 @@ crc_status crc_cache_update(const crc_bank* bank, const crc_shape* shape, int32_
   return e == cudaSuccess ? CRC_OK : cuda_fail(e);
 }
 
+size_t crc_retrieve_workspace_size(int32_t bank_count, int32_t k) {
+  if (bank_count < 0 || k < 1 || k > CRC_MAX_K) return 0;
+  return crc::retrieve_workspace_bytes(bank_count, k);
+}
+
 crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shape* shape, const crc_frame* cur,
                         int32_t n, const crc_retrieval* p, const crc_cache* cache, const crc_rope* rope,
-                        int32_t* d_idx, double* d_score, int32_t* d_count, cudaStream_t s) {
+                        int32_t* d_idx, double* d_score, int32_t* d_count, void* d_workspace, size_t workspace_bytes,
+                        cudaStream_t s) {
   CRC_RANGE("crc_retrieve");
   crc_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_bank(bank, cache != nullptr))) return st;
   if (!cur || !p || !d_idx || !d_count) return CRC_ERR_INVALID_ARG;
   if (bank_count < 0 || bank_count > bank->capacity || n < 0) return CRC_ERR_INVALID_ARG;
-  if (p->k < 1 || p->k > CRC_MAX_K || !(p->E > 0.0) || isnan(p->w_v) || isnan(p->tau_c) || isnan(p->cos_tau_v))
+  if (p->k < 1 || p->k > CRC_MAX_K || !(p->E > 0.0) || !isfinite(p->E) || !isfinite(p->w_v) || isnan(p->tau_c) ||
+      isnan(p->cos_tau_v))
     return CRC_ERR_INVALID_ARG;
   if (!frames_ok(cur, shape->F)) return CRC_ERR_INVALID_ARG;
+  const size_t ws = crc::retrieve_workspace_bytes(bank_count, p->k);
+  if (ws > 0 && (!d_workspace || workspace_bytes < ws || !aligned16(d_workspace))) return CRC_ERR_INVALID_ARG;
   crc::RetrieveArgs a;
   memset(&a, 0, sizeof(a));
   pack_frames(a.cur, cur, shape->F);
   a.centre = bank->centre;
   a.view = bank->view;
+  a.slab_chunk = bank->slab_chunk;
+  a.num_slabs = bank->num_slabs;
+  if (ws > 0) {
+    a.partial = static_cast<crc::TopkCand*>(d_workspace);
+    a.ticket = reinterpret_cast<unsigned int*>(static_cast<char*>(d_workspace) + ws - 256);
+  }
   a.count = bank_count;
   a.n = n;
   a.E = p->E;
@@ -283,9 +299,11 @@ crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shap
   a.d_score = d_score;
   a.d_count = d_count;
   if ((st = check_rope(rope, shape))) return st;
-  a.g.pool = nullptr;
-  if (cache && (st = fill_gather(a.g, shape, bank->kv, bank->num_slabs, cache, p->k, rope))) return st;
-  cudaError_t e = crc::launch_retrieve(a, s);
+  crc::GatherArgs g;
+  memset(&g, 0, sizeof(g));
+  g.pool = nullptr;
+  if (cache && (st = fill_gather(g, shape, bank->kv, bank->num_slabs, cache, p->k, rope))) return st;
+  cudaError_t e = crc::launch_retrieve(a, g, s);
   return e == cudaSuccess ? CRC_OK : cuda_fail(e);
 }
 
@@ -351,7 +369,8 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
   if (n_q != nc) return CRC_ERR_SHAPE;
   if (k < 0 || k > CRC_MAX_K || !isfinite(lambda) || lambda < 0.f || !(sigma > 0.f) || !isfinite(sigma))
     return CRC_ERR_INVALID_ARG;
-  if (flags & ~(CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN | CRC_ATTN_SKIP_FAR)) return CRC_ERR_INVALID_ARG;
+  if (flags & ~(CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN | CRC_ATTN_SKIP_FAR | CRC_ATTN_BIAS_DIRECT))
+    return CRC_ERR_INVALID_ARG;
   bool any_ret = false, any_other = false;
   for (int g = 0; g < cache->nseg; ++g) {
     if (cache->seg[g].kind == CRC_SEG_RETRIEVED && cache->seg[g].length > 0) {
@@ -362,6 +381,8 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
     }
   }
   if (any_ret && (!d_uv || !d_valid)) return CRC_ERR_INVALID_ARG;
+  // the kernels read each correspondence as one float2
+  if (((uintptr_t)d_uv & 7u) != 0) return CRC_ERR_UNSUPPORTED;
   if (q.stride_head < shape->d || q.stride_token < (int64_t)shape->H * q.stride_head ||
       o.stride_head < shape->d || o.stride_token < (int64_t)shape->H * o.stride_head)
     return CRC_ERR_SHAPE;
@@ -400,6 +421,7 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
   a.dtype = shape->dtype;
   a.status = d_status;
   a.bias_form = (flags & CRC_ATTN_GAUSSIAN) ? 1 : 0;
+  a.bias_direct = (flags & CRC_ATTN_BIAS_DIRECT) ? 1 : 0;
   // skipped weights are scaled by at most 2^-64: lambda d^2 / (2 sigma^2) >= 64 ln 2
   a.skip_far = (flags & CRC_ATTN_SKIP_FAR) && !(flags & CRC_ATTN_GAUSSIAN) && lambda > 0.f && any_ret && any_other &&
                        d_valid
@@ -416,6 +438,10 @@ crc_status crc_biased_attention(const crc_shape* shape, crc_tensor q, const crc_
     if (e == cudaErrorNotSupported) return CRC_ERR_UNSUPPORTED;
   }
   return e == cudaSuccess ? CRC_OK : cuda_fail(e);
+}
+
+double crc_bias_expansion_bound(float lambda, float sigma, int32_t h, int32_t w) {
+  return crc::bias_expansion_bound(lambda, sigma, h, w);
 }
 
 }  // extern "C"

@@ -54,10 +54,22 @@
 // rescaled only on those rare steps.  Keys outside every segment and retrieved
 // slots without a chunk produce no tile at all.
 //
+// Accuracy of the expansion.  Its large terms (A q_k, 2 A ux' x'_k, ...) cancel to
+// A d^2 near the correspondence, so its absolute error grows with the grid: in base-2
+// logit units it stays below 2^-23 C (w^2 + h^2), C = lambda log2(e) / (2 sigma^2).
+// The error comes from rounding the query coefficients -2A ux', -2A uy' and
+// A (ux'^2 + uy'^2) to fp32 before their (exact) three-term split: a CPU model of
+// those steps alone gives 0.43-0.67 x 2^-24 C (w^2 + h^2), and this GPU measures
+// 0.49-0.64 of that unit, so the tensor core's fp32 sum adds little.  The key terms
+// are exact for grids up to 256 a side with (w-1)^2 + (h-1)^2 < 2^16.  Where the
+// bound exceeds 2^-9 -- the bf16 rounding of P -- or the grid is larger, the host
+// selects the direct form (MODE = DIRECT): the K = 16 operand carries only the mask
+// and the softmax adds C d^2 to every biased score from the key's cell, exact to
+// fp32 rounding, at a lower throughput.
+//
 // The opt-in additive-Gaussian form (lambda exp(-d^2 / (2 sigma^2)) on the same
-// columns) has no low-rank expansion.  Its instantiation (GAUSS = true) keeps only
-// the mask in the K = 16 operand and adds the bonus to S in the softmax, column by
-// column, before the row max.
+// columns) has no low-rank expansion either: its instantiation (MODE = GAUSS) adds
+// the bonus to S in the softmax, column by column, before the row max.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -256,9 +268,15 @@ __device__ __forceinline__ void fail(const TcParams& P, volatile int* abort_flag
 
 }  // namespace
 
-// GAUSS: the opt-in additive-Gaussian bias form (CRC_ATTN_GAUSSIAN); the Eq. 2
-// instantiation carries none of its code.
-template <bool GAUSS>
+// How the bias reaches S: the Eq. 2 expansion on the tensor core, or per score in
+// the softmax (Eq. 2 directly, or the opt-in additive-Gaussian form).
+constexpr int kBiasTensor = 0;
+constexpr int kBiasGauss = 1;
+constexpr int kBiasDirect = 2;
+
+// MODE: one of the kBias* forms; the tensor-core instantiation carries none of the
+// per-score code.
+template <int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ TcParams P) {
@@ -459,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = 2 * bt + h;
         const uint32_t mask = row <= (int)ti.nact_m1 ? 0u : neg;
         uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, mask << 16};
-        if (ti.s >= 0 && !GAUSS) {
+        if (ti.s >= 0 && MODE == kBiasTensor) {
           // grid cell of the key inside its source frame, relative to the frame centre
           const int loc = (int)ti.loc0 + row;
           const int yi = loc / a.w;
@@ -632,9 +650,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // loaded one tile ahead so that the global-load latency overlaps a tile
     Corr nxt = load_corr(a, tiles, 0, nt, p, row_ok, P.coef_log2);
     // query-side bias/mask operand: the first tile's source frame (or no bias).  In
-    // the additive-Gaussian form it carries only the mask multiplier, and the bonus
-    // is added to S in the softmax from the current frame's correspondence `cur`.
-    constexpr bool gauss = GAUSS;
+    // the per-score forms it carries only the mask multiplier, and the bias is added
+    // to S in the softmax from the current frame's correspondence `cur`.
+    constexpr bool gauss = MODE != kBiasTensor;
     const Corr none{0.f, 0.f, 0.f};
     int aug_frame = nt > 0 ? tiles[0].s : -1;
     Corr cur = nxt;
@@ -663,28 +681,35 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32u * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
       tmem_wait_ld();
-      if constexpr (GAUSS) {
-        // additive-Gaussian form: S += lambda sqrt(d) 2^(-d^2 log2(e) / (2 sigma^2)) for a
-        // biased tile and a valid correspondence, with d the grid distance from the key's
-        // cell (x, y), walked column by column, to u^ of the tile's source frame
+      if constexpr (MODE != kBiasTensor) {
+        // per-score bias for a biased tile and a valid correspondence, with d the grid
+        // distance from the key's cell (x, y), walked column by column, to u^ of the
+        // tile's source frame:
+        //   GAUSS:  S += lambda sqrt(d) 2^(-d^2 log2(e) / (2 sigma^2))
+        //   DIRECT: S += (C / scale) d^2, Eq. 2 in raw score units (C < 0)
         const TileInfo tj = tiles[j];
         if (tj.s >= 0 && cur.cA != 0.f) {
           const int y0 = (int)tj.loc0 / a.w;
           float xf = (float)((int)tj.loc0 - y0 * a.w), yf = (float)y0;
           const float wf = (float)a.w, gk = P.gauss_k, gc = P.gauss_gc;
+          const float araw = cur.cA * inv_sc;
           float dy = cur.uyA - yf;
-          float dy2k = dy * dy * gk;
+          float dy2 = MODE == kBiasGauss ? dy * dy * gk : dy * dy;
 #pragma unroll
           for (int c = 0; c < 128; ++c) {
             const float dx = cur.uxA - xf;
-            const float g = ex2(-fmaf(dx * dx, gk, dy2k));
-            sr[c] = __float_as_uint(fmaf(gc, g, __uint_as_float(sr[c])));
+            if constexpr (MODE == kBiasGauss) {
+              const float g = ex2(-fmaf(dx * dx, gk, dy2));
+              sr[c] = __float_as_uint(fmaf(gc, g, __uint_as_float(sr[c])));
+            } else {
+              sr[c] = __float_as_uint(fmaf(araw, fmaf(dx, dx, dy2), __uint_as_float(sr[c])));
+            }
             xf += 1.f;
             if (xf == wf) {
               xf = 0.f;
               yf += 1.f;
               dy = cur.uyA - yf;
-              dy2k = dy * dy * gk;
+              dy2 = MODE == kBiasGauss ? dy * dy * gk : dy * dy;
             }
           }
         }
@@ -817,6 +842,14 @@ bool make_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void*
 
 }  // namespace
 
+double bias_expansion_bound(float lambda, float sigma, int h, int w) {
+  // the key operand holds x', y' (half-integers up to (w-1)/2) and q = x'^2 + y'^2 (two
+  // terms) exactly in bf16 only while 2|x'|, 2|y'| < 256 and 4q < 2^16
+  if (w > 256 || h > 256 || (int64_t)(w - 1) * (w - 1) + (int64_t)(h - 1) * (h - 1) >= 65536) return INFINITY;
+  const double C = (double)lambda * 1.4426950408889634 / (2.0 * (double)sigma * (double)sigma);
+  return C * ((double)w * w + (double)h * h) * 0x1p-23;
+}
+
 cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
   if (a.dtype != CRC_BF16 || a.d != HD) return cudaErrorNotSupported;
   int64_t ntiles = 0;  // the kernel's tiling: per segment, per frame for retrieved segments
@@ -854,7 +887,10 @@ cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
   P.gauss_gc = (float)((double)a.lambda * sqrt((double)a.d));
   P.gauss_k = (float)(1.4426950408889634 / (2.0 * (double)a.sigma * (double)a.sigma));
   P.timeout_ns = 2000000000ull;
-  auto kernel = a.bias_form != 0 ? attn_tc_kernel<true> : attn_tc_kernel<false>;
+  auto kernel = a.bias_form == 1 ? attn_tc_kernel<kBiasGauss>
+                : (a.bias_direct || bias_expansion_bound(a.lambda, a.sigma, a.h, a.w) > kExpansionLimit)
+                    ? attn_tc_kernel<kBiasDirect>
+                    : attn_tc_kernel<kBiasTensor>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
   dim3 grid((a.Nq + NQT * BM - 1) / (NQT * BM), a.H, a.L);

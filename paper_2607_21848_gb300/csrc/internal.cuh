@@ -53,11 +53,29 @@ struct PoseInsertArgs {
 };
 cudaError_t launch_pose_summary(const PoseInsertArgs& a, cudaStream_t s);
 
+// Per-step values of crc_chunk_step, read on the device.  A launcher given a step
+// takes the chunk index, window offset, fallback chunk, re-positioning target,
+// segment lengths and frames from it instead of its own arguments.
+using StepDesc = crc_step;
+static_assert(sizeof(crc_frame) == 21 * sizeof(double), "crc_frame is 21 packed doubles");
+
 struct CacheUpdateArgs {
+  const StepDesc* step;    // crc_chunk_step: chunk, window offset, frames and the pointers below
+  int32_t* status;         // set to CRC_STEP_BAD_DESCRIPTOR for a descriptor out of range
+  int32_t capacity;        // bank chunks (descriptor check)
+  int32_t num_slabs;
+  int64_t slab_bytes;
+  char* kv_base;           // bank->kv
+  int32_t* slab_chunk;     // bank->slab_chunk or null
+  float* depth_base;       // bank->depth
+  char* cache_k;           // cache bases (window slot derived from the descriptor)
+  char* cache_v;
+  int32_t n_keys;
   FrameSet frames;
   double* bank_frames;
   double* bank_centre;
   double* bank_view;
+  int32_t* slab_owner;     // bank->slab_chunk + chunk % num_slabs, or null
   int32_t chunk;
   const float* depth_src;  // [F][h][w]
   float* depth_dst;        // bank depth + chunk * F*h*w
@@ -93,16 +111,29 @@ struct GatherArgs {
   int32_t d;            // head dim
   int32_t elem_bytes;   // 2 (bf16) or 4 (fp32)
   int32_t F;
+  const StepDesc* step;  // crc_chunk_step: rope_pos_slot0 from the descriptor
   // rope (rope_pairs = 0: plain copy)
   int32_t rope_pairs, rope_c0, rope_interleaved;
   int32_t rope_pos_slot0, rope_pos_stride, rope_frame_pos0;
   double rope_omega[CRC_MAX_ROPE_PAIRS];  // theta^(-i/pairs)
 };
 
+// One candidate of the top-k: the score as an order-preserving 64-bit key, and j.
+struct TopkCand {
+  unsigned long long key;
+  int32_t j;
+  int32_t pad;
+};
+
 struct RetrieveArgs {
+  const StepDesc* step;  // crc_chunk_step: n, count = n + 1, ext_first and frames from the descriptor
+  int32_t* status;       // descriptor check (with a step)
+  int32_t capacity;
   FrameSet cur;
   const double* centre;
   const double* view;
+  const int32_t* slab_chunk;  // [num_slabs] chunk held by each K/V slab, or null (no residency test)
+  int32_t num_slabs;
   int32_t count;
   int32_t n;
   double E, w_v, tau_c, cos_tau_v;
@@ -110,18 +141,25 @@ struct RetrieveArgs {
   int32_t* d_idx;
   double* d_score;
   int32_t* d_count;
-  GatherArgs g;
+  TopkCand* partial;     // [grid][k] per-block candidates (workspace; null with one block)
+  unsigned int* ticket;  // blocks done (workspace; zeroed before the launch)
 };
-cudaError_t launch_retrieve(const RetrieveArgs& a, cudaStream_t s);
+
+// Blocks and workspace bytes of the top-k launch over `count` bank entries.
+int retrieve_blocks(int32_t count);
+size_t retrieve_workspace_bytes(int32_t count, int32_t k);
 
 struct GatherOnlyArgs {
   const int32_t* d_idx;  // [k] chunk per slot (negative = empty)
   int32_t k;
   GatherArgs g;
 };
-cudaError_t launch_gather(const GatherOnlyArgs& a, cudaStream_t s);
+// The top-k launch, then (g.pool non-null) the gather launch that reads its d_idx.
+cudaError_t launch_retrieve(const RetrieveArgs& a, const GatherArgs& g, cudaStream_t s);
+cudaError_t launch_gather(const GatherOnlyArgs& a, cudaStream_t s, bool after_topk = false);
 
 struct CorrespondArgs {
+  const StepDesc* step;      // crc_chunk_step: the current frames from the descriptor
   FrameSet cur;
   const float* depth;        // [F][h][w]
   const double* bank_frames; // [capacity][F][21]
@@ -138,6 +176,7 @@ struct CorrespondArgs {
 cudaError_t launch_correspond(const CorrespondArgs& a, cudaStream_t s);
 
 struct AttnArgs {
+  const StepDesc* step;  // crc_chunk_step: segment lengths from the descriptor (at most seg[].length)
   const void* q;
   const void* k;
   const void* v;
@@ -158,11 +197,26 @@ struct AttnArgs {
   int32_t dtype;
   int32_t* status;
   int32_t bias_form;  // 0: Eq. 2 quadratic; 1: additive Gaussian (CRC_ATTN_GAUSSIAN)
+  int32_t bias_direct;  // Eq. 2 evaluated per score even where the tensor-core expansion is accurate
   int32_t skip_far;   // CRC_ATTN_SKIP_FAR in force (tensor-core kernel)
   float skip_d2;      // squared grid distance beyond which a retrieved tile is skipped
 };
+// Length of cache segment g in this call: the descriptor's, clamped to the plan's.
+// A retrieved segment is all or nothing (N_c keys or none).
+__device__ __forceinline__ int32_t seg_length(const AttnArgs& a, int g) {
+  const int32_t len = a.seg[g].length;
+  if (a.step == nullptr) return len;
+  const int32_t sl = a.step->seg_length[g];
+  if (a.seg[g].kind == CRC_SEG_RETRIEVED) return sl > 0 ? len : 0;
+  return sl < 0 ? 0 : (sl < len ? sl : len);
+}
+
 cudaError_t launch_attn_simt(const AttnArgs& a, cudaStream_t s);
 // Returns cudaErrorNotSupported when the tensor-core kernel cannot take these arguments.
 cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s);
+// Error bound of the tensor-core expansion of Eq. 2, in base-2 logit units, and the
+// bound above which the tensor-core kernel evaluates Eq. 2 per score instead.
+double bias_expansion_bound(float lambda, float sigma, int h, int w);
+constexpr double kExpansionLimit = 0x1p-9;
 
 }  // namespace crc

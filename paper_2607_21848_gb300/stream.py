@@ -3,7 +3,8 @@
 Cache layout (Sec. 4.2): [sink | retrieved slot 0 .. k-1 | window ring 0 .. W-1],
 each region one chunk (N_c tokens) long.  The first chunk becomes the sink and is
 never evicted; chunk n >= 1 goes into window ring slot n % W, evicting the chunk
-W steps older; every chunk stays in the bank.  One step n runs, on one stream and
+W steps older; every chunk's poses and depth stay in the bank, and its K/V as long as
+its slab (chunk % num_slabs) is not reused.  One step n runs, on one stream and
 without any host synchronisation:
 
   crc_cache_update    chunk n's K/V, depth and poses enter the window and the bank
@@ -45,7 +46,7 @@ class StreamConfig:
     k: int
     window: int  # chunks in the recent window (the current chunk included)
     capacity: int  # chunks the bank can hold
-    num_slabs: int
+    num_slabs: int  # K/V slabs; with fewer than `capacity`, only the newest num_slabs chunks can be retrieved
     E: float
     w_v: float
     tau_c: float
@@ -79,7 +80,10 @@ class ChunkStream:
         self.cfg = cfg
         c = cfg
         self.shape = api.shape(c.L, c.H, c.d, c.F, c.h, c.w, c.dtype)
-        self.bank = api.Bank(c.capacity, c.F, c.h, c.w, c.L, c.H, c.d, c.dtype, c.num_slabs, device=device)
+        # the bank records which chunk each K/V slab holds: with fewer slabs than chunks, a chunk
+        # whose slab a newer chunk overwrote is never retrieved
+        self.bank = api.Bank(c.capacity, c.F, c.h, c.w, c.L, c.H, c.d, c.dtype, c.num_slabs, device=device,
+                             track_slabs=True)
         self.cache = api.Cache.empty(c.L, c.n_keys, c.H, c.d, c.dtype, [], device=device)
         self.idx = torch.full((c.k,), -1, dtype=torch.int32, device=device)
         self.score = torch.zeros(c.k, dtype=torch.float64, device=device)
@@ -95,7 +99,7 @@ class ChunkStream:
             # the control branch keeps its own slab pool and cache; poses and depth live in the main bank
             self.control_shape = api.shape(c.control_L, c.H, c.d, c.F, c.h, c.w, c.dtype)
             self.control_bank = api.Bank(c.capacity, c.F, c.h, c.w, c.control_L, c.H, c.d, c.dtype, c.num_slabs,
-                                         device=device)
+                                         device=device, track_slabs=True)
             self.control_cache = api.Cache.empty(c.control_L, c.n_keys, c.H, c.d, c.dtype, [], device=device)
 
     # ---- checkpoint -------------------------------------------------------
@@ -104,7 +108,7 @@ class ChunkStream:
         slabs), the cache and, if present, the control branch's pool and cache.  The
         step index is the caller's (segments and ring slots follow from it).  The
         tensors are the stream's own; save or clone them before stepping on."""
-        sd = {"bank." + k: getattr(self.bank, k) for k in ("frames", "centre", "view", "depth", "kv")}
+        sd = {"bank." + k: getattr(self.bank, k) for k in ("frames", "centre", "view", "depth", "kv", "slab_chunk")}
         sd["cache.k"], sd["cache.v"] = self.cache.k, self.cache.v
         if self.control_shape is not None:
             sd["control_bank.kv"] = self.control_bank.kv

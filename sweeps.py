@@ -1,8 +1,11 @@
 """Stand-alone sweeps of single kernels, for measurement and profiling (e.g. under ncu):
 
-  python -m paper_2607_21848_gb300.sweeps correspond      # 126 MB reprojection sweep, scene depth
-  python -m paper_2607_21848_gb300.sweeps correspond-iid  # the same with depth drawn per token
-  python -m paper_2607_21848_gb300.sweeps gather       # crc_gather, plain and re-positioned
+  python sweeps.py correspond      # 126 MB reprojection sweep, scene depth
+  python sweeps.py correspond-iid  # the same with depth drawn per token
+  python sweeps.py gather          # crc_gather, plain and re-positioned
+
+Measurement tooling beside bench.py (which imports it for its context block); not part
+of the library package.
 """
 
 from __future__ import annotations
@@ -134,7 +137,7 @@ def main(argv=None):
     what = argv[0] if argv else "correspond"
     import os
 
-    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))  # the synth package
+    sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))  # the package and the synth module
     from paper_2607_21848_gb300 import build
 
     build.build()

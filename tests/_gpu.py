@@ -27,7 +27,7 @@ def oracle_bank_poses(fr: synth.Frames):
     return c, v
 
 
-def oracle_retrieve(wl, bank_count=None, n=None, k=None, ext_first=-1, ext_min=0, **over):
+def oracle_retrieve(wl, bank_count=None, n=None, k=None, ext_first=-1, ext_min=0, resident=None, **over):
     fr = wl.bank_frames
     B = fr.shape[0] if bank_count is None else bank_count
     bc, bv = oracle_bank_poses(fr[:B])
@@ -36,8 +36,8 @@ def oracle_retrieve(wl, bank_count=None, n=None, k=None, ext_first=-1, ext_min=0
     p = dict(E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c, cos_tau_v=wl.cos_tau_v, delta=wl.delta)
     p.update(over)
     n = wl.n if n is None else n
-    idx, score, count = oracle.retrieve(bc, bv, cn, vn, n, k=wl.k if k is None else k, **p)
-    slots = oracle.fill_slots(idx, count, ext_first, ext_min)
+    idx, score, count = oracle.retrieve(bc, bv, cn, vn, n, k=wl.k if k is None else k, resident=resident, **p)
+    slots = oracle.fill_slots(idx, count, ext_first, ext_min, resident=resident)
     return idx, score, count, slots
 
 

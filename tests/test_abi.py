@@ -59,7 +59,7 @@ _LAYOUT_C = r"""
 #define O(T, f) printf(#T "." #f " %zu\n", offsetof(T, f));
 int main(void) {
   P(crc_frame) P(crc_shape) P(crc_tensor) P(crc_segment) P(crc_cache) P(crc_bank) P(crc_retrieval) P(crc_rope)
-  O(crc_cache, v) O(crc_cache, n_keys) O(crc_cache, seg) O(crc_bank, frames) O(crc_bank, kv)
+  O(crc_cache, v) O(crc_cache, n_keys) O(crc_cache, seg) O(crc_bank, frames) O(crc_bank, kv) O(crc_bank, slab_chunk)
   O(crc_retrieval, delta) O(crc_retrieval, ext_min) O(crc_retrieval, exclude_sink) O(crc_shape, dtype)
   O(crc_tensor, stride_head) O(crc_rope, frame_pos0) O(crc_rope, theta)
   return 0;
@@ -89,7 +89,8 @@ def test_ctypes_layout_matches_header():
         "crc_rope.frame_pos0": _abi.crc_rope.frame_pos0.offset, "crc_rope.theta": _abi.crc_rope.theta.offset,
         "crc_cache.v": _abi.crc_cache.v.offset, "crc_cache.n_keys": _abi.crc_cache.n_keys.offset,
         "crc_cache.seg": _abi.crc_cache.seg.offset, "crc_bank.frames": _abi.crc_bank.frames.offset,
-        "crc_bank.kv": _abi.crc_bank.kv.offset, "crc_retrieval.delta": _abi.crc_retrieval.delta.offset,
+        "crc_bank.kv": _abi.crc_bank.kv.offset,
+        "crc_bank.slab_chunk": _abi.crc_bank.slab_chunk.offset, "crc_retrieval.delta": _abi.crc_retrieval.delta.offset,
         "crc_retrieval.ext_min": _abi.crc_retrieval.ext_min.offset, "crc_shape.dtype": _abi.crc_shape.dtype.offset,
         "crc_tensor.stride_head": _abi.crc_tensor.stride_head.offset,
     }
@@ -129,4 +130,4 @@ def test_retrieve_rejects_a_negative_chunk_index(lib):
         frames[f].R[:] = [1.0, 0.0, 0.0, 0.0, 1.0, 0.0, 0.0, 0.0, 1.0]
     params = _abi.crc_retrieval(1.0, 0.5, float("inf"), -1.0, 1, 1, -1, 0, 0)
     assert lib.crc_retrieve(C.byref(bank), 4, C.byref(shape), frames, -1, C.byref(params), None, None, fake, None,
-                            fake, None) == _abi.CRC_ERR_INVALID_ARG
+                            fake, None, 0, None) == _abi.CRC_ERR_INVALID_ARG

@@ -48,9 +48,11 @@ def _frames(n=F, **bad):
 
 
 def _bank(**over):
-    v = dict(capacity=8, num_slabs=4, frames=_ptr(1), centre=_ptr(2), view=_ptr(3), depth=_ptr(4), kv=_ptr(5))
+    v = dict(capacity=8, num_slabs=4, frames=_ptr(1), centre=_ptr(2), view=_ptr(3), depth=_ptr(4), kv=_ptr(5),
+             slab_chunk=None)
     v.update(over)
-    return _abi.crc_bank(v["capacity"], v["num_slabs"], v["frames"], v["centre"], v["view"], v["depth"], v["kv"])
+    return _abi.crc_bank(v["capacity"], v["num_slabs"], v["frames"], v["centre"], v["view"], v["depth"], v["kv"],
+                         v["slab_chunk"])
 
 
 def _segments(k=1, window=2):
@@ -136,29 +138,55 @@ def test_cache_update_rejections(lib, case, status):
 
 
 # ---- crc_retrieve and crc_gather ---------------------------------------------------------------
-@pytest.mark.parametrize("params", [_params(E=0.0), _params(E=-1.0), _params(k=0), _params(k=_abi.CRC_MAX_K + 1),
-                                    _params(w_v=math.nan), _params(tau_c=math.nan), _params(cos_tau_v=math.nan)])
+@pytest.mark.parametrize("params", [_params(E=0.0), _params(E=-1.0), _params(E=math.inf), _params(k=0),
+                                    _params(k=_abi.CRC_MAX_K + 1), _params(w_v=math.nan), _params(w_v=math.inf),
+                                    _params(tau_c=math.nan), _params(cos_tau_v=math.nan)])
 def test_retrieve_rejects_bad_parameters(lib, params):
     sh, b, c = _shape(), _bank(), _cache()
     assert lib.crc_retrieve(C.byref(b), 8, C.byref(sh), _frames(), 5, C.byref(params), C.byref(c), None, _ptr(11),
-                            None, _ptr(12), None) == INVALID
+                            None, _ptr(12), None, 0, None) == INVALID
 
 
 def test_retrieve_rejects_bad_counts_and_outputs(lib):
     sh, b, c, p = _shape(), _bank(), _cache(), _params()
     call = lambda count, n=5, idx=_ptr(11), cnt=_ptr(12): lib.crc_retrieve(  # noqa: E731
-        C.byref(b), count, C.byref(sh), _frames(), n, C.byref(p), C.byref(c), None, idx, None, cnt, None)
+        C.byref(b), count, C.byref(sh), _frames(), n, C.byref(p), C.byref(c), None, idx, None, cnt, None, 0, None)
     assert call(9) == INVALID          # bank_count > capacity
     assert call(-1) == INVALID
     assert call(8, idx=None) == INVALID
     assert call(8, cnt=None) == INVALID
 
 
+def test_retrieve_workspace_size_and_rejections(lib):
+    size = lib.crc_retrieve_workspace_size
+    assert size(512, 8) == 0 and size(0, 1) == 0          # one block: no workspace
+    assert size(513, 1) > 0                                  # two blocks meet in the workspace
+    assert size(100000, 3) <= size(100000, 8) <= size(10 ** 9, 8) < 300 * 1024
+    assert size(2000, 0) == 0 and size(2000, _abi.CRC_MAX_K + 1) == 0 and size(-1, 1) == 0
+    sh, c, p = _shape(), _cache(), _params(k=3)
+    b = _bank(capacity=4096)
+    need = size(4096, 3)
+    call = lambda ws, nbytes: lib.crc_retrieve(  # noqa: E731
+        C.byref(b), 4096, C.byref(sh), _frames(), 4096, C.byref(p), C.byref(c), None, _ptr(11), None, _ptr(12), ws,
+        nbytes, None)
+    assert call(None, 0) == INVALID                  # a bank of 4096 needs a workspace
+    assert call(_ptr(20), need - 16) == INVALID      # too short
+    assert call(_ptr(20) + 8, need) == INVALID       # not 16-byte aligned
+
+
+def test_bank_slab_owner_needs_the_slab_pool(lib):
+    # an owner array describes the K/V slabs: without a pool the bank is rejected
+    sh, c, p = _shape(), _cache(), _params()
+    b = _bank(kv=None, slab_chunk=_ptr(21))
+    assert lib.crc_retrieve(C.byref(b), 8, C.byref(sh), _frames(), 5, C.byref(p), None, None, _ptr(11), None,
+                            _ptr(12), None, 0, None) == INVALID
+
+
 def test_retrieve_and_gather_reject_two_segments_for_one_slot(lib):
     sh, b, p = _shape(), _bank(), _params()
     dup = _cache([(0, NC, _abi.CRC_SEG_RETRIEVED, 0), (NC, NC, _abi.CRC_SEG_RETRIEVED, 0)], 2 * NC)
     assert lib.crc_retrieve(C.byref(b), 8, C.byref(sh), _frames(), 5, C.byref(p), C.byref(dup), None, _ptr(11), None,
-                            _ptr(12), None) == SHAPE
+                            _ptr(12), None, 0, None) == SHAPE
     assert lib.crc_gather(C.byref(sh), _ptr(5), 4, _ptr(11), 1, C.byref(dup), None, None) == SHAPE
 
 
@@ -234,11 +262,12 @@ def test_attention_rejects_bad_parameters(lib):
     assert _attend(lib, sigma=math.inf) == INVALID
     assert _attend(lib, k=-1) == INVALID
     assert _attend(lib, k=_abi.CRC_MAX_K + 1) == INVALID
-    assert _attend(lib, flags=8) == INVALID             # unknown flag bit
+    assert _attend(lib, flags=16) == INVALID            # unknown flag bit
     assert _attend(lib, uv=None) == INVALID             # retrieved segments need correspondences
     assert _attend(lib, valid=None) == INVALID
     assert _attend(lib, k=0) == SHAPE                   # a retrieved segment's slot must be < k
     assert _attend(lib, q_stride_head=d - 8) == SHAPE   # heads of q overlap
+    assert _attend(lib, uv=_ptr(13) + 4) == UNSUPPORTED  # correspondences are read as float2
 
 
 def test_attention_rejects_bad_segment_tables(lib):

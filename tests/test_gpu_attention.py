@@ -89,6 +89,37 @@ def _check_bf16_peaky(Og, Oo, Oabs):
     assert worst <= 1.0, worst
 
 
+def _ulp_bf16(x):
+    a = np.maximum(np.abs(x), 2.0 ** -126)
+    return 2.0 ** (np.floor(np.log2(a)) - 7)
+
+
+def _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, lam, sigma, bias="tensor"):
+    """The tensor-core output against a CPU model of the kernel's own rounding steps
+    (tests/_tc_model.py: tiles cut per segment and frame, the stale row max, P rounded to
+    bf16 at the kernel's scale, the expansion's coefficients as the kernel rounds them).
+    The kernel must reproduce the model bit for bit in almost every element.  What is left
+    are fp32-level differences (the tensor core's summation order, ex2.approx) that now and
+    then move a weight across a bf16 rounding boundary: one such flip changes P by 2^-8 of
+    one weight, so O by at most 2^-9 sum_k w_k |v_k| (one bf16 ulp of O besides).  The
+    kernel's error against the oracle must then be the model's error plus that slack plus
+    the expansion's stated bound carried through the softmax weights."""
+    from tests import _tc_model as model
+
+    F, h, w, k = geom
+    Om, _ = model.attention_model(Q, Kc, Vc, uv, valid, segs, h, w, F, lam, sigma, bias=bias)
+    Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, lam, sigma)
+    dm = np.abs(Og - Om)
+    slack = _ulp_bf16(Om) + 2.0 ** -9 * Oabs
+    assert (dm == 0).mean() >= 0.99, (dm == 0).mean()
+    assert (dm <= slack).all(), float((dm / slack).max())
+    eb = api.crc_bias_expansion_bound(lam, sigma, h, w) if bias == "tensor" else 0.0
+    bound = np.abs(Om - Oo) + slack + math.log(2) * eb * (Oabs + np.abs(Oo)) + 1e-6
+    err = np.abs(Og - Oo)
+    assert (err <= bound).all(), float((err / bound).max())
+    assert err.max() <= 2e-2
+
+
 def test_fp32_tiny_8x8_matches_oracle_1e4():
     wl = synth.make_workload(1)
     idx, _, count, slots = _gpu.oracle_retrieve(wl)
@@ -121,8 +152,8 @@ def test_bf16_tcgen05_small_ragged(lam, sigma):
     (1, 8, 8, 2, False),    # a chunk of 64 queries: less than one query tile
     (3, 5, 26, 1, False),   # 130-token frames: a full tile and a 2-key tail per frame
     # the most frames and slots: 32 source frames of 60 tokens, a new query-side bias operand
-    # on every KV tile.  Single rows reach 6x the output RMS, so the bound is the bf16
-    # rounding of P and O per element rather than 2e-2 x RMS.
+    # on every KV tile.  Single rows reach 6x the output RMS, so 2e-2 x RMS is below the bf16
+    # rounding of P and O there: the check is the kernel's own rounding model instead.
     (4, 6, 10, 8, True),
 ])
 def test_bf16_tcgen05_frame_shapes(F, h, w, k, peaky):
@@ -130,8 +161,7 @@ def test_bf16_tcgen05_frame_shapes(F, h, w, k, peaky):
     Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, k, 4.0, 1.0)
     Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 4.0, 1.0)
     if peaky:
-        Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, 4.0, 1.0)
-        _check_bf16_peaky(Og, Oo, Oabs)
+        _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, 4.0, 1.0)
         assert np.abs(lg - lo).max() <= 1e-3
         Og2, _ = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, k, 4.0, 1.0)
         np.testing.assert_array_equal(Og, Og2)  # deterministic
@@ -212,8 +242,10 @@ def test_bf16_maximum_tile_count_and_one_key_beyond():
     assert bool((o == 7.0).all())
 
 
-def _full_size(cfg, rows, layers, heads, seed=7):
+def _full_size(cfg, rows, layers, heads, seed=7, lam=None, sigma=None, flags=0):
     wl = synth.make_workload(cfg)
+    lam = wl.lam if lam is None else lam
+    sigma = wl.sigma if sigma is None else sigma
     _, _, count, slots = _gpu.oracle_retrieve(wl)
     uv, _, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
     uv = uv.astype(np.float32)
@@ -224,18 +256,19 @@ def _full_size(cfg, rows, layers, heads, seed=7):
     kc = (torch.randn(wl.L, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
     vc = (torch.randn(wl.L, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
     shp = api.shape(wl.L, wl.H, wl.d, wl.F, wl.h, wl.w, torch.bfloat16)
-    Og, lg = _run_attn(shp, q, kc, vc, wl.segments, uv, valid, wl.k, wl.lam, wl.sigma, slot_chunk=slots)
+    Og, lg = _run_attn(shp, q, kc, vc, wl.segments, uv, valid, wl.k, lam, sigma, slot_chunk=slots, flags=flags)
     Lsel, Hsel = list(layers), list(heads)
     Qo = q[Lsel][:, :, Hsel].float().cpu().numpy()
     Ko = kc[Lsel][:, :, Hsel].float().cpu().numpy()
     Vo = vc[Lsel][:, :, Hsel].float().cpu().numpy()
-    Oo, lo = oracle.attention(Qo, Ko, Vo, uv.astype(np.float64), valid, wl.segments, wl.h, wl.w, wl.F, wl.lam,
-                              wl.sigma, slot_chunks=slots, rows=rows)
+    Oo, lo = oracle.attention(Qo, Ko, Vo, uv.astype(np.float64), valid, wl.segments, wl.h, wl.w, wl.F, lam,
+                              sigma, slot_chunks=slots, rows=rows)
     Og = Og[Lsel][:, :, Hsel]
     lg = lg[Lsel][:, Hsel]
     _check_bf16(Og, lg, Oo, lo, rows=rows)
     # the correspondence bias changes the output by far more than the tolerance
     assert valid.mean() > 0.05
+    return Og if rows is None else Og[:, rows]
 
 
 def test_bf16_wan13b_chunk_full_size_sampled_rows():
@@ -262,6 +295,89 @@ def test_bf16_14b_720p_full_size_sampled():
     rows = np.random.default_rng(2).choice(10800, 512, replace=False)
     rows.sort()
     _full_size(4, rows, [0], range(40))
+
+
+# ---------------------------------------------------------------------------- accuracy of the tensor-core bias
+def _lse_probe(h, w, lam, sigma, flags=0, rows=None, seed=0):
+    """Q = 0 against one retrieved frame of h x w keys: the row's LSE is log sum exp(lambda B)
+    alone, so its error is the bias error on the keys that carry the row's weight.
+    Correspondences are spread over the whole grid, the four corners included."""
+    g = np.random.default_rng(seed)
+    Nc = h * w
+    cx, cy = g.integers(0, w, Nc), g.integers(0, h, Nc)
+    cx[:4], cy[:4] = [0, w - 1, 0, w - 1], [0, 0, h - 1, h - 1]
+    uv = np.stack([cx + g.uniform(-0.5, 0.5, Nc), cy + g.uniform(-0.5, 0.5, Nc)], -1)[:, None, :].astype(np.float32)
+    valid = np.ones((Nc, 1), bool)
+    segs = [(0, Nc, api.SEG_RETRIEVED, 0)]
+    zeros = np.zeros((1, Nc, 1, 128), np.float32)
+    shp = api.shape(1, 1, 128, 1, h, w, torch.bfloat16)
+    _, lg = _run_attn(shp, zeros, zeros, zeros, segs, uv, valid, 1, lam, sigma, flags=flags)
+    rows = np.arange(Nc) if rows is None else rows
+    _, lo = oracle.attention(zeros, zeros, zeros, uv.astype(np.float64), valid, segs, h, w, 1, lam, sigma, rows=rows)
+    # error and magnitude in base-2 units; fp32 rounding of the per-score arithmetic, the LSE
+    # and the row sum, relative to the magnitude of the bias that carries the row
+    err = np.abs(lg[0, 0, rows] - lo[0, 0]) / math.log(2)
+    return err, 2.0 ** -20 * np.maximum(np.abs(lo[0, 0]) / math.log(2), 1.0)
+
+
+@pytest.mark.parametrize("h,w,lam,sigma", [(12, 16, 8.0, 0.5), (30, 52, 2.0, 1.0), (30, 52, 4.0, 1.0),
+                                           (45, 80, 2.0, 1.0), (45, 80, 2.69, 1.0), (90, 160, 0.6, 1.0)])
+def test_bias_expansion_error_is_within_its_stated_bound(h, w, lam, sigma):
+    """On the tensor-core expansion (these settings are within its 2^-9 limit), the measured
+    bias error stays below crc_bias_expansion_bound; the per-score form is exact to fp32."""
+    bound = api.crc_bias_expansion_bound(lam, sigma, h, w)
+    assert bound <= 2.0 ** -9
+    rows = None if h * w <= 4000 else np.arange(0, h * w, 7)
+    err, fp32 = _lse_probe(h, w, lam, sigma, rows=rows)
+    assert (err <= bound + fp32).all(), (err.max(), bound)
+    assert err.max() >= 0.1 * bound  # the probe does see the expansion's error
+    err_d, fp32 = _lse_probe(h, w, lam, sigma, flags=api.ATTN_BIAS_DIRECT, rows=rows)
+    assert (err_d <= fp32).all(), err_d.max()
+
+
+@pytest.mark.parametrize("h,w,lam,sigma", [(45, 80, 8.0, 0.5), (30, 52, 32.0, 0.5), (12, 300, 2.0, 1.0)])
+def test_steep_biases_and_wide_grids_take_the_per_score_form(h, w, lam, sigma):
+    """Beyond the expansion's limit (or where its key terms are not exact in bf16) the kernel
+    evaluates Eq. 2 per score: the LSE error is at the fp32 level, not the expansion's."""
+    assert api.crc_bias_expansion_bound(lam, sigma, h, w) > 2.0 ** -9
+    rows = np.arange(0, h * w, 11)
+    err, fp32 = _lse_probe(h, w, lam, sigma, rows=rows)
+    assert (err <= fp32).all(), err.max()
+
+
+def test_bf16_14b_grid_steep_bias_full_size_sampled():
+    """The 14B-class 720p shape (45 x 80 grid, 40 heads, 64 800 keys) with the steepest bias of
+    the tests, lambda = 8 and sigma = 0.5 (per-score form): sampled rows of every head."""
+    rows = np.random.default_rng(3).choice(10800, 384, replace=False)
+    rows.sort()
+    _full_size(4, rows, [0], range(40), lam=8.0, sigma=0.5)
+
+
+def test_bf16_14b_grid_steepest_tensor_core_bias_full_size_sampled():
+    """The same shape with the steepest bias the tensor-core expansion takes on a 45 x 80 grid
+    (lambda / sigma^2 = 2.69, just inside its 2^-9 limit): sampled rows of every head."""
+    assert api.crc_bias_expansion_bound(2.69, 1.0, 45, 80) <= 2.0 ** -9
+    rows = np.random.default_rng(4).choice(10800, 384, replace=False)
+    rows.sort()
+    _full_size(4, rows, [0], range(40), lam=2.69, sigma=1.0)
+
+
+def test_bias_direct_flag_agrees_with_the_expansion_at_the_wan13b_shape():
+    """CRC_ATTN_BIAS_DIRECT at the Wan-1.3B chunk shape (one layer): both forms within the
+    tolerance of the oracle, and within bf16 rounding of each other."""
+    rows = np.random.default_rng(5).choice(4680, 512, replace=False)
+    rows.sort()
+    Ot = _full_size(2, rows, [0], range(12))
+    Od = _full_size(2, rows, [0], range(12), flags=api.ATTN_BIAS_DIRECT)
+    err, rel, _ = _gpu.attn_errors(Ot, Od.astype(np.float64))
+    assert err <= 2e-2 and rel <= 4e-2
+
+
+def test_bf16_direct_form_follows_the_kernel_model_on_32_source_frames():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=11 + 4 + 6, L=1, H=2, F=4, h=6, w=10, k=8)
+    Og, _ = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, 8, 4.0, 1.0, flags=api.ATTN_BIAS_DIRECT)
+    Oo, _ = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 4.0, 1.0)
+    _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, 4.0, 1.0, bias="direct")
 
 
 # ---------------------------------------------------------------------------- opt-in modes
@@ -329,7 +445,7 @@ def test_gaussian_form_tensor_core_full_size_sampled_and_against_simt():
 def test_unknown_attention_flags_are_rejected():
     shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=22, L=1, H=1)
     with pytest.raises(api.CrcError):
-        _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=8)
+        _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=16)
 
 
 def _skip_case(seed, far_logit=0.0, invalid_row=None):

@@ -79,6 +79,112 @@ def test_retrieve_gates_bit_exact(over):
     np.testing.assert_array_equal(gs, os_)
 
 
+def _random_bank(B, seed, ties=0):
+    """B entries with random centres and unit view directions; with `ties`, runs of
+    entries share one pose (identical scores) spread over the whole bank."""
+    g = np.random.default_rng(seed)
+    c = g.normal(size=(B, 3)) * 20.0
+    v = g.normal(size=(B, 3))
+    v /= np.linalg.norm(v, axis=1, keepdims=True)
+    pos = np.zeros(3)
+    if ties:  # the tied entries share the pose of a camera at c[pick[0]] looking along +x
+        pick = g.choice(B, ties, replace=False)
+        pos = c[pick[0]].copy()
+        c[pick] = pos
+        v[pick] = [1.0, 0.0, 0.0]
+    return c, v, pos
+
+
+@pytest.mark.parametrize("B,k,ties", [(513, 3, 0), (4097, 8, 0), (100003, 3, 0), (100003, 8, 0), (20000, 8, 40)])
+def test_retrieve_large_banks_bit_exact(B, k, ties):
+    """Banks of more than 512 entries are scored by many blocks whose candidates meet in the
+    workspace: indices, count and fp64 scores bit-exact against the oracle, ties across
+    blocks broken by the chunk index, and every gate in force."""
+    c, v, pos = _random_bank(B, seed=B + k, ties=ties)
+    bank = api.Bank(B, 3, 8, 8, 1, 1, 64, torch.float32, 1, with_kv=False)
+    bank.centre.copy_(torch.from_numpy(c))
+    bank.view.copy_(torch.from_numpy(v))
+    assert bank.workspace is not None
+    shp = api.shape(1, 1, 64, 3, 8, 8, torch.float32)
+    K = synth.pinhole(8, 8, 90.0)
+    # the current chunk looks along +x from the tied pose (or the origin)
+    cur = synth.Frames(np.stack([K] * 3), np.stack([synth.camera_rotation(0.0)] * 3), np.stack([pos] * 3))
+    cn, vn = oracle.chunk_pose(cur.R, cur.c)
+    for over in (dict(E=10.0, w_v=0.5, tau_c=math.inf, cos_tau_v=-1.0, delta=1),
+                 dict(E=10.0, w_v=0.5, tau_c=3.0, cos_tau_v=math.cos(math.radians(60)), delta=B // 3)):
+        n = B + 5
+        oi, os_, oc = oracle.retrieve(c, v, cn, vn, n, k=k, **over)
+        params = api.retrieval_params(over["E"], over["w_v"], over["tau_c"], over["cos_tau_v"], over["delta"], k)
+        idx = torch.full((k,), -7, dtype=torch.int32, device="cuda")
+        score = torch.zeros(k, dtype=torch.float64, device="cuda")
+        count = torch.full((1,), -7, dtype=torch.int32, device="cuda")
+        api.crc_retrieve(bank, B, shp, synth.frame_records(cur), n, params, None, idx, score, count)
+        torch.cuda.synchronize()
+        assert int(count.item()) == oc
+        np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+        np.testing.assert_array_equal(score.cpu().numpy(), os_)
+        if ties and math.isinf(over["tau_c"]):
+            assert oc == k and len(set(os_[:k])) == 1  # k equal scores (0), ordered by j
+
+
+def test_retrieve_admits_only_chunks_whose_slab_still_holds_them():
+    """A bank of 12 chunks with a pool of 4 tracked K/V slabs: after 12 updates only the
+    last 4 chunks are held.  Retrieval admits only those (the oracle over the resident
+    chunks), the window-extension fallback skips chunks that are no longer held, and the
+    gathered K/V are each chunk's own."""
+    F, h, w, L, H, d, P, B = 3, 8, 8, 1, 2, 64, 4, 12
+    Nc = F * h * w
+    K = synth.pinhole(h, w, 90.0)
+    fr = synth.random_walk(synth.rng(77, "poses"), B, F, K, step=0.3, radius=3.0)
+    shp = api.shape(L, H, d, F, h, w, torch.float32)
+    bank = api.Bank(B, F, h, w, L, H, d, torch.float32, P, track_slabs=True)
+    g = torch.Generator(device="cuda").manual_seed(9)
+    kv = [(torch.randn(L, Nc, H, d, generator=g, device="cuda"), torch.randn(L, Nc, H, d, generator=g, device="cuda"))
+          for _ in range(B)]
+    depth = torch.ones(F, h, w, device="cuda")
+    for j in range(B):
+        api.crc_cache_update(bank, shp, j, synth.frame_records(fr[j]), depth, kv[j][0], kv[j][1], None, -1)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(bank.slab_chunk.cpu().numpy(), [8, 9, 10, 11])
+    resident = np.zeros(B, bool)
+    resident[B - P:] = True
+    bc, bv = _gpu.oracle_bank_poses(fr)
+    cur = fr[3]
+    cn, vn = oracle.chunk_pose(cur.R, cur.c)
+    k = 3
+    segs = [(0, Nc, api.SEG_SINK, 0)] + [((1 + r) * Nc, Nc, api.SEG_RETRIEVED, r) for r in range(k)]
+    for n, delta, ext_first in ((B, 1, -1), (B, 5, 9), (B, 3, 10)):  # [8..11] top-3; [9, 8, -]; [8, 9] + 10
+        oi, os_, oc = oracle.retrieve(bc, bv, cn, vn, n, 1.0, 0.5, math.inf, -1.0, delta, k, resident=resident)
+        slots = oracle.fill_slots(oi, oc, ext_first, 1, resident=resident)
+        cache = api.Cache.empty(L, (1 + k) * Nc, H, d, torch.float32, segs)
+        params = api.retrieval_params(1.0, 0.5, math.inf, -1.0, delta, k, ext_first, 1)
+        idx = torch.full((k,), -7, dtype=torch.int32, device="cuda")
+        count = torch.zeros(1, dtype=torch.int32, device="cuda")
+        api.crc_retrieve(bank, B, shp, synth.frame_records(cur), n, params, cache, idx, None, count)
+        torch.cuda.synchronize()
+        gi = idx.cpu().numpy()
+        assert int(count.item()) == oc
+        np.testing.assert_array_equal(gi, slots)
+        assert all(resident[j] for j in gi if j >= 0)
+        for r, j in enumerate(gi):
+            if j >= 0:
+                off = (1 + r) * Nc
+                assert torch.equal(cache.k[:, off:off + Nc], kv[j][0])
+                assert torch.equal(cache.v[:, off:off + Nc], kv[j][1])
+    # without the owner array every chunk is admissible (the caller vouches for the slabs)
+    untracked = api.Bank(B, F, h, w, L, H, d, torch.float32, P)
+    untracked.centre.copy_(bank.centre)
+    untracked.view.copy_(bank.view)
+    oi, _, oc = oracle.retrieve(bc, bv, cn, vn, B, 1.0, 0.5, math.inf, -1.0, 1, k)
+    idx = torch.full((k,), -7, dtype=torch.int32, device="cuda")
+    count = torch.zeros(1, dtype=torch.int32, device="cuda")
+    api.crc_retrieve(untracked, B, shp, synth.frame_records(cur), B,
+                     api.retrieval_params(1.0, 0.5, math.inf, -1.0, 1, k), None, idx, None, count)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    assert not all(resident[j] for j in oi)  # the sub-bank and the whole bank differ here
+
+
 def test_retrieve_stream_gates_and_window_extension():
     wl = synth.make_workload(5)
     bank, shp = _gpu.make_bank(wl, torch.bfloat16)

@@ -2,8 +2,10 @@
 Wan-1.3B head shape, 30 layers, k = 2) through ChunkStream: every step's
 retrieval must match the oracle bit-exactly and its correspondences within the
 boundary band; the cache invariants (sink = chunk 0, window = newest chunks,
-retrieved slots = their slabs) must hold; attention is compared with the oracle on
-sampled steps, layers and query rows."""
+retrieved slots = the retrieved chunks' own K/V) must hold; attention is compared
+with the oracle on sampled steps, layers and query rows.  The bank keeps the K/V of
+all 200 chunks (200 slabs, 172 GB at 30 layers); a second stream with a pool of 16
+slabs checks that a chunk whose slab was reused is never retrieved."""
 
 import numpy as np
 import pytest
@@ -26,7 +28,7 @@ def _built():
 def test_loop_stream_200_steps():
     wl = synth.make_workload(5)
     cfg = crs.StreamConfig(L=wl.L, H=wl.H, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2,
-                           capacity=wl.bank_size, num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c,
+                           capacity=wl.bank_size, num_slabs=wl.bank_size, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c,
                            cos_tau_v=wl.cos_tau_v, delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps)
     st = crs.ChunkStream(cfg)
     Nc = cfg.Nc
@@ -43,10 +45,6 @@ def test_loop_stream_200_steps():
     host_kv = [(kb[layers][:, :, heads].double().cpu().numpy(), vb[layers][:, :, heads].double().cpu().numpy())
                for kb, vb in kv_new]
     host_q = q[layers][:, :, heads].double().cpu().numpy()
-
-    def slab_owner(slab, n):
-        """Newest chunk m <= n written to K/V slab `slab` (chunk m lives in slab m % P)."""
-        return slab + ((n - slab) // cfg.num_slabs) * cfg.num_slabs
     n_closed = 0
     for n in range(wl.bank_size):
         fr = wl.bank_frames[n]
@@ -70,9 +68,9 @@ def test_loop_stream_200_steps():
             assert torch.equal(st.cache.k[:, off:off + Nc], kv_new[m % nbuf][0])
             assert torch.equal(st.cache.v[:, off:off + Nc], kv_new[m % nbuf][1])
         for r, j in enumerate(slots):
-            if j >= 0:
+            if j >= 0:  # the retrieved chunk's own K/V (chunk j was written from buffer j % nbuf)
                 off = st.slot_offset(r)
-                src = kv_new[slab_owner(j % cfg.num_slabs, n) % nbuf]
+                src = kv_new[j % nbuf]
                 assert torch.equal(st.cache.k[:, off:off + Nc], src[0])
                 assert torch.equal(st.cache.v[:, off:off + Nc], src[1])
         # correspondences
@@ -93,7 +91,7 @@ def test_loop_stream_200_steps():
             for rr, j in enumerate(slots):
                 if j >= 0:
                     off = st.slot_offset(rr)
-                    Kx[:, off:off + Nc], Vx[:, off:off + Nc] = host_kv[slab_owner(j % cfg.num_slabs, n) % nbuf]
+                    Kx[:, off:off + Nc], Vx[:, off:off + Nc] = host_kv[j % nbuf]
             for m in range(max(1, n - 1), n + 1):
                 off = st.window_offset(m % 2)
                 Kx[:, off:off + Nc], Vx[:, off:off + Nc] = host_kv[m % nbuf]
@@ -108,6 +106,50 @@ def test_loop_stream_200_steps():
             lg = lse[layers][:, heads].cpu().numpy()[:, :, rows]
             assert np.abs(lg - lo).max() <= 1e-3
     assert n_closed >= 40  # the loop closes after one lap and stays closed
+    del st
+    torch.cuda.empty_cache()
+
+
+def test_loop_stream_with_a_small_slab_pool_never_gathers_a_reused_slab():
+    """The same 200-step loop with 16 K/V slabs for 200 chunks (2 layers, 2 heads): chunk j's
+    slab is reused by chunk j + 16, so from then on j is not retrievable.  Every step's
+    retrieval equals the oracle's over the chunks still held, and every gathered slot holds
+    its chunk's own K/V."""
+    wl = synth.make_workload(5)
+    P = 16
+    cfg = crs.StreamConfig(L=2, H=2, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2, capacity=wl.bank_size,
+                           num_slabs=P, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c, cos_tau_v=wl.cos_tau_v,
+                           delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps)
+    st = crs.ChunkStream(cfg)
+    Nc = cfg.Nc
+    g = torch.Generator(device="cuda").manual_seed(12)
+    kv = [((torch.randn(2, Nc, 2, cfg.d, generator=g, device="cuda") * wl.qkv_scale).bfloat16(),
+           (torch.randn(2, Nc, 2, cfg.d, generator=g, device="cuda") * wl.qkv_scale).bfloat16()) for _ in range(5)]
+    q = kv[0][0].clone()
+    o = torch.empty_like(q)
+    closed_full = closed_held = 0
+    for n in range(wl.bank_size):
+        kn, vn = kv[n % 5]
+        st.step(n, synth.frame_records(wl.bank_frames[n]), torch.from_numpy(wl.depth_of(n)).cuda(), kn, vn, q, o)
+        torch.cuda.synchronize()
+        assert st.status.item() == 0
+        held = np.zeros(wl.bank_size, bool)
+        held[max(0, n - P + 1):n + 1] = True
+        _, _, oc, slots = _gpu.oracle_retrieve(wl, bank_count=n + 1, n=n, ext_first=st.ext_first(n), ext_min=1,
+                                               resident=held)
+        gi = st.idx.cpu().numpy()
+        assert int(st.count.item()) == oc, n
+        np.testing.assert_array_equal(gi, slots)
+        for r, j in enumerate(gi):
+            if j >= 0:
+                assert held[j]
+                off = st.slot_offset(r)
+                assert torch.equal(st.cache.k[:, off:off + Nc], kv[j % 5][0])
+                assert torch.equal(st.cache.v[:, off:off + Nc], kv[j % 5][1])
+        closed_held += oc > 0
+        closed_full += _gpu.oracle_retrieve(wl, bank_count=n + 1, n=n)[2] > 0
+    # the loop's start (chunks 0-2) is long gone from the 16-slab pool when the camera returns
+    assert closed_full >= 40 and closed_held < closed_full
 
 
 def test_loop_stream_with_rope_repositioning_and_control_mirror():
@@ -115,7 +157,7 @@ def test_loop_stream_with_rope_repositioning_and_control_mirror():
     # mirroring the retrieved slots (small head count; retrieval and gathers are what is checked)
     wl = synth.make_workload(5)
     cfg = crs.StreamConfig(L=2, H=2, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2, capacity=wl.bank_size,
-                           num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c, cos_tau_v=wl.cos_tau_v,
+                           num_slabs=wl.bank_size, E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c, cos_tau_v=wl.cos_tau_v,
                            delta=wl.delta, lam=wl.lam, sigma=wl.sigma, eps=wl.eps, rope_pairs=22,
                            rope_interleaved=True, control_L=1)
     st = crs.ChunkStream(cfg)
@@ -131,9 +173,6 @@ def test_loop_stream_with_rope_repositioning_and_control_mirror():
     ctl = [(rnd(1), rnd(1)) for _ in range(nbuf)]
     q = rnd(cfg.L)
     o = torch.empty_like(q)
-
-    def slab_owner(slab, n):
-        return slab + ((n - slab) // cfg.num_slabs) * cfg.num_slabs
 
     def rope_of(n):
         r = st.rope(n)
@@ -160,7 +199,7 @@ def test_loop_stream_with_rope_repositioning_and_control_mirror():
         for r, j in enumerate(slots):
             if j < 0:
                 continue
-            owner = slab_owner(j % cfg.num_slabs, n) % nbuf
+            owner = j % nbuf  # chunk j's own K/V
             off = st.slot_offset(r)
             for cache, src in ((st.cache, kv[owner]), (st.control_cache, ctl[owner])):
                 host = np.stack([src[0].double().cpu().numpy(), src[1].double().cpu().numpy()])
@@ -178,8 +217,8 @@ def test_stream_resumes_from_a_checkpoint_bit_for_bit(tmp_path):
     # run 30 steps; checkpoint after step 19 to a file; a fresh stream restored from it
     # replays steps 20-29 with identical retrievals, correspondences and outputs
     wl = synth.make_workload(5)
-    cfg = crs.StreamConfig(L=2, H=2, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2, capacity=wl.bank_size,
-                           num_slabs=wl.num_slabs, E=wl.E, w_v=wl.w_v, tau_c=1.0, cos_tau_v=-1.0, delta=wl.delta,
+    cfg = crs.StreamConfig(L=2, H=2, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2, capacity=30,
+                           num_slabs=16, E=wl.E, w_v=wl.w_v, tau_c=1.0, cos_tau_v=-1.0, delta=wl.delta,
                            lam=wl.lam, sigma=wl.sigma, eps=wl.eps, rope_pairs=22, control_L=1)
     g = torch.Generator(device="cuda").manual_seed(8)
 

@@ -139,6 +139,33 @@ def test_empty_admissible_set_extends_window():
     assert list(oracle.fill_slots(idx, 0, ext_first=-1, ext_min=1)) == [-1, -1]
 
 
+def test_retrieval_over_resident_chunks_equals_retrieval_over_that_sub_bank():
+    # a chunk whose keys and values are no longer held is not admissible: the result is that of
+    # Eq. 1 over the bank with those chunks removed (brute force on the sub-bank, indices mapped back)
+    g = np.random.default_rng(8)
+    bc = g.normal(size=(40, 3)) * 4
+    bv = g.normal(size=(40, 3))
+    bv /= np.linalg.norm(bv, axis=1, keepdims=True)
+    cn, vn = g.normal(size=3), np.array([0.0, 1.0, 0.0])
+    resident = g.uniform(size=40) < 0.5
+    args = (cn, vn, 100, 2.0, 0.5, math.inf, -1.0, 1, 6)
+    idx, score, count = oracle.retrieve(bc, bv, *args, resident=resident)
+    keep = np.nonzero(resident)[0]
+    idx2, score2, count2 = oracle.retrieve(bc[keep], bv[keep], *args)
+    assert count == count2 == 6
+    assert list(idx) == list(keep[idx2])
+    np.testing.assert_array_equal(score, score2)
+    assert resident[idx[:count]].all()
+    # every chunk resident: the literal Eq. 1
+    full = oracle.retrieve(bc, bv, *args)
+    assert list(oracle.retrieve(bc, bv, *args, resident=np.ones(40, bool))[0]) == list(full[0])
+    # the window-extension fallback skips a chunk that is no longer held
+    res = np.ones(10, bool)
+    res[6] = False
+    assert list(oracle.fill_slots(np.array([-1, -1], dtype=np.int32), 0, 7, 1, resident=res)) == [7, -1]
+    assert list(oracle.fill_slots(np.array([-1, -1], dtype=np.int32), 0, 6, 1, resident=res)) == [-1, 5]
+
+
 def test_gather_is_slab_copy():
     pool = np.arange(4 * 2 * 1 * 3 * 1 * 2, dtype=np.float32).reshape(4, 2, 1, 3, 1, 2)
     out = oracle.gather(pool, np.array([5, -1, 2]), 4)
