@@ -418,14 +418,29 @@ typedef struct {
   int32_t* d_cell;           /* [N_c][k F] or NULL                                             */
   uint8_t* d_valid;          /* [N_c][k F]                                                     */
   int32_t* d_status;         /* [1], required: CRC_STEP_BAD_DESCRIPTOR when a kernel finds the
-                                descriptor out of range (it then writes nothing else), or a
-                                pipeline timeout code of the attention kernel                   */
+                                descriptor out of range (the bank and the cache are then left
+                                untouched, the retrieval reports no chunk and the step's
+                                outputs are not valid), or a timeout code of the attention kernel */
   void* d_workspace;         /* crc_retrieve_workspace_size(bank.capacity, k) bytes            */
   size_t workspace_bytes;
 } crc_step_plan;
 
 #define CRC_STEP_BAD_DESCRIPTOR 100
 
+/*
+ * crc_chunk_step — one chunk step with the per-step values of *d_step: the same
+ * results, bit for bit, as crc_cache_update(bank, shape, n, frames, d_depth, d_k,
+ * d_v, cache, window_offset), crc_retrieve over chunks 0..n (ext_first and the
+ * re-positioning from the descriptor), crc_correspond and crc_biased_attention with
+ * the descriptor's segment lengths, in that order on stream s.  Everything in the
+ * plan is validated on the host; the descriptor is checked on the device (n within
+ * the bank, the window slot within the cache, segment lengths within the plan's).
+ * Enqueued work: the K/V and pose update, a 4-byte memset (when the retrieval
+ * workspace is used), the scoring, the gather, the reprojection and the attention.
+ * Errors: as the four calls, and CRC_ERR_INVALID_ARG for a missing status word,
+ * descriptor or workspace.
+ */
+crc_status crc_chunk_step(const crc_step_plan* plan, const crc_step* d_step, cudaStream_t s);
 
 /* Bound on the error of the tensor-core expansion of the Eq. 2 bias on an h x w grid,
  * in base-2 logit units: 2^-23 lambda log2(e) / (2 sigma^2) (w^2 + h^2); +inf where

@@ -76,6 +76,24 @@ class crc_rope(C.Structure):
                 ("pos_stride", C.c_int32), ("frame_pos0", C.c_int32), ("theta", C.c_double)]
 
 
+class crc_step(C.Structure):
+    _fields_ = [("n", C.c_int32), ("window_offset", C.c_int32), ("ext_first", C.c_int32),
+                ("rope_pos_slot0", C.c_int32), ("seg_length", C.c_int32 * CRC_MAX_SEGMENTS),
+                ("frames", crc_frame * CRC_MAX_FRAMES)]
+
+
+class crc_step_plan(C.Structure):
+    _fields_ = [("shape", crc_shape), ("bank", crc_bank), ("cache", crc_cache), ("retrieval", crc_retrieval),
+                ("rope", crc_rope), ("eps", C.c_float), ("lam", C.c_float), ("sigma", C.c_float),
+                ("attn_flags", C.c_int32), ("d_depth", C.c_void_p), ("d_k", C.c_void_p), ("d_v", C.c_void_p),
+                ("q", crc_tensor), ("o", crc_tensor), ("d_lse", C.c_void_p), ("d_idx", C.c_void_p),
+                ("d_score", C.c_void_p), ("d_count", C.c_void_p), ("d_uv", C.c_void_p), ("d_cell", C.c_void_p),
+                ("d_valid", C.c_void_p), ("d_status", C.c_void_p), ("d_workspace", C.c_void_p),
+                ("workspace_bytes", C.c_size_t)]
+
+
+CRC_STEP_BAD_DESCRIPTOR = 100
+
 _P = C.POINTER
 _SIGS = {
     "crc_version": (C.c_char_p, []),
@@ -97,6 +115,7 @@ _SIGS = {
                                          C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_float, C.c_float,
                                          C.c_int32, C.c_void_p, C.c_void_p]),
     "crc_bias_expansion_bound": (C.c_double, [C.c_float, C.c_float, C.c_int32, C.c_int32]),
+    "crc_chunk_step": (C.c_int32, [_P(crc_step_plan), C.c_void_p, C.c_void_p]),
 }
 
 EXPORTED = tuple(_SIGS)

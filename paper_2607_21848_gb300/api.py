@@ -141,6 +141,14 @@ def rope_params(channel0: int, pairs: int, theta: float, interleaved: bool, pos_
     return _abi.crc_rope(channel0, pairs, int(bool(interleaved)), pos_slot0, pos_stride, frame_pos0, float(theta))
 
 
+def crc_chunk_step(plan: _abi.crc_step_plan, d_step: torch.Tensor, stream=None) -> None:
+    """One chunk step with its per-step values read from the device descriptor d_step
+    (a uint8 tensor holding one crc_step)."""
+    if d_step.numel() * d_step.element_size() < C.sizeof(_abi.crc_step):
+        raise ValueError("d_step is smaller than a crc_step")
+    _abi.check("crc_chunk_step", _abi.load().crc_chunk_step(C.byref(plan), _ptr(d_step), _stream(stream)))
+
+
 def crc_bias_expansion_bound(lam: float, sigma: float, h: int, w: int) -> float:
     return float(_abi.load().crc_bias_expansion_bound(lam, sigma, h, w))
 

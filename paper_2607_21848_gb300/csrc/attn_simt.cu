@@ -134,8 +134,10 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const __grid_constant__ 
   }
 }
 
+bool attn_simt_supported(const AttnArgs& a) { return a.d <= kMaxD && (a.d % 32) == 0; }
+
 cudaError_t launch_attn_simt(const AttnArgs& a, cudaStream_t s) {
-  if (a.d > kMaxD || (a.d % 32) != 0) return cudaErrorNotSupported;
+  if (!attn_simt_supported(a)) return cudaErrorNotSupported;
   dim3 grid((a.Nq + kQB - 1) / kQB, a.H, a.L);
   if (a.dtype == CRC_F32)
     attn_simt_kernel<float><<<grid, 128, 0, s>>>(a);

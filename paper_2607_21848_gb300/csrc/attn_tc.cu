@@ -353,13 +353,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     int count = 0, qa = 0;
     for (int g = 0; g < a.nseg; ++g) {
       const crc_segment sg = a.seg[g];
-      if (sg.length <= 0) continue;
+      const int len = seg_length(a, g);
+      if (len <= 0) continue;
       const bool ret = sg.kind == CRC_SEG_RETRIEVED;
       if (ret && a.slot_chunk && a.slot_chunk[sg.slot] < 0) continue;  // empty slot: masked
       const int nr = ret ? a.F : 1;
       for (int rr = 0; rr < nr; ++rr) {
         const int rstart = ret ? sg.offset + rr * hw : sg.offset;
-        const int rlen = ret ? hw : sg.length;
+        const int rlen = ret ? hw : len;
         const int ntile = (rlen + BN - 1) / BN;
         for (int base = 0; base < ntile; base += 32) {
           const int t = base + lane;
@@ -850,9 +851,12 @@ double bias_expansion_bound(float lambda, float sigma, int h, int w) {
   return C * ((double)w * w + (double)h * h) * 0x1p-23;
 }
 
-cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
-  if (a.dtype != CRC_BF16 || a.d != HD) return cudaErrorNotSupported;
-  int64_t ntiles = 0;  // the kernel's tiling: per segment, per frame for retrieved segments
+// The kernel's limits: bf16, d = 128, at most kMaxTiles KV tiles (each segment cut
+// from its start, a retrieved one per frame; the largest segment lengths count),
+// S <= 127 source frames, h w <= 65535, 16-byte aligned tensors and strides, sm_103.
+bool attn_tc_supported(const AttnArgs& a) {
+  if (a.dtype != CRC_BF16 || a.d != HD) return false;
+  int64_t ntiles = 0;
   for (int g = 0; g < a.nseg; ++g) {
     const crc_segment& sg = a.seg[g];
     if (sg.length <= 0) continue;
@@ -861,17 +865,21 @@ cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
     else
       ntiles += (sg.length + BN - 1) / BN;
   }
-  if (ntiles > kMaxTiles || a.S > 127 || a.h * a.w > 65535) return cudaErrorNotSupported;
+  if (ntiles > kMaxTiles || a.S > 127 || a.h * a.w > 65535) return false;
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
-  if (!al16(a.q) || !al16(a.k) || !al16(a.v) || !al16(a.o)) return cudaErrorNotSupported;
+  if (!al16(a.q) || !al16(a.k) || !al16(a.v) || !al16(a.o)) return false;
   const int64_t strides[9] = {a.q_sl, a.q_st, a.q_sh, a.k_sl, a.k_st, a.k_sh, a.o_sl, a.o_st, a.o_sh};
   for (int64_t x : strides)
-    if ((x * 2) % 16 != 0) return cudaErrorNotSupported;
+    if ((x * 2) % 16 != 0) return false;
   int dev = 0, major = 0, minor = 0;
-  cudaGetDevice(&dev);
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-  if (major != 10 || minor != 3) return cudaErrorNotSupported;
+  return major == 10 && minor == 3;
+}
+
+cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
+  if (!attn_tc_supported(a)) return cudaErrorNotSupported;
   auto enc = tensor_map_encoder();
   if (!enc) return cudaErrorNotSupported;
   CUtensorMap mq, mk, mv;

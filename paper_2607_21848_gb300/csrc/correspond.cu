@@ -132,7 +132,7 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   // data that grid may write (indices, bank records, depths) or writes outputs.
   if (i < nt) {
     const int t = t_lo + i;
-    const double* ft = &a.cur.rec[t][0];
+    const double* ft = a.step ? reinterpret_cast<const double*>(&a.step->frames[t]) : &a.cur.rec[t][0];
     float Kt[9], Rt[9], Ki[9];
     for (int e = 0; e < 9; ++e) {
       Kt[e] = f64_to_f32(ft[e]);

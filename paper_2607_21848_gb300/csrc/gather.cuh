@@ -22,17 +22,17 @@ struct GatherPlan {
 };
 
 // Position shift of slot r holding chunk j: from frame_pos0 + j*F to pos_slot0 + r*pos_stride.
-__device__ __forceinline__ int64_t rope_delta(const GatherArgs& g, int r, int64_t j) {
-  return (int64_t)g.rope_pos_slot0 + (int64_t)r * g.rope_pos_stride - ((int64_t)g.rope_frame_pos0 + j * g.F);
+__device__ __forceinline__ int64_t rope_delta(const GatherArgs& g, int32_t pos_slot0, int r, int64_t j) {
+  return (int64_t)pos_slot0 + (int64_t)r * g.rope_pos_stride - ((int64_t)g.rope_frame_pos0 + j * g.F);
 }
 
 // Fills plan.rotate[] and plan.cs[] once plan.chunk[] is visible to the whole block.
 // Angles are formed in fp64 (delta * omega_i) so that large position shifts keep
 // their accuracy; the rotation itself runs in fp32.  Ends with a block barrier.
-__device__ inline void plan_rope(const GatherArgs& g, int k, GatherPlan& p) {
+__device__ inline void plan_rope(const GatherArgs& g, int k, GatherPlan& p, int32_t pos_slot0) {
   for (int r = threadIdx.x; r < k; r += blockDim.x) {
     const int64_t j = p.chunk[r];
-    p.rotate[r] = (g.rope_pairs > 0 && j >= 0 && rope_delta(g, r, j) != 0) ? 1 : 0;
+    p.rotate[r] = (g.rope_pairs > 0 && j >= 0 && rope_delta(g, pos_slot0, r, j) != 0) ? 1 : 0;
   }
   const int n = k * g.rope_pairs;
   for (int e = threadIdx.x; e < n; e += blockDim.x) {
@@ -40,7 +40,7 @@ __device__ inline void plan_rope(const GatherArgs& g, int k, GatherPlan& p) {
     const int64_t j = p.chunk[r];
     if (j < 0) continue;
     double sn, cn;
-    sincos((double)rope_delta(g, r, j) * g.rope_omega[i], &sn, &cn);
+    sincos((double)rope_delta(g, pos_slot0, r, j) * g.rope_omega[i], &sn, &cn);
     p.cs[r][i] = make_float2((float)cn, (float)sn);
   }
   __syncthreads();

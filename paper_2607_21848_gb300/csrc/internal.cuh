@@ -212,8 +212,10 @@ __device__ __forceinline__ int32_t seg_length(const AttnArgs& a, int g) {
 }
 
 cudaError_t launch_attn_simt(const AttnArgs& a, cudaStream_t s);
-// Returns cudaErrorNotSupported when the tensor-core kernel cannot take these arguments.
 cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s);
+// Whether a kernel can take these arguments (checked on the host before any launch).
+bool attn_simt_supported(const AttnArgs& a);
+bool attn_tc_supported(const AttnArgs& a);
 // Error bound of the tensor-core expansion of Eq. 2, in base-2 logit units, and the
 // bound above which the tensor-core kernel evaluates Eq. 2 per score instead.
 double bias_expansion_bound(float lambda, float sigma, int h, int w);

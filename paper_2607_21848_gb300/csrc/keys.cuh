@@ -19,7 +19,7 @@ __device__ __forceinline__ KeyInfo key_info_of(const AttnArgs& a, int key) {
   if (key >= a.Nk) return ki;
   for (int g = 0; g < a.nseg; ++g) {
     const crc_segment sg = a.seg[g];
-    if (key < sg.offset || key >= sg.offset + sg.length) continue;
+    if (key < sg.offset || key >= sg.offset + seg_length(a, g)) continue;
     if (sg.kind == CRC_SEG_RETRIEVED) {
       if (a.slot_chunk && a.slot_chunk[sg.slot] < 0) return ki;  // empty slot: masked
       const int hw = a.h * a.w;

@@ -160,9 +160,29 @@ __global__ void __launch_bounds__(kTopkThreads) retrieve_topk_kernel(const __gri
   const int tid = threadIdx.x;
   // let the gather grid begin its launch; it waits for this grid's results
   asm volatile("griddepcontrol.launch_dependents;");
+  // the current chunk, the bank entries and the fallback: the arguments', or a step descriptor's
+  int n = a.n, count = a.count, ext_first = a.ext_first;
+  const double* cur = &a.cur.rec[0][0];
+  if (a.step) {
+    n = a.step->n;
+    if (n < 0 || n >= a.capacity) {  // every block sees the same descriptor
+      if (blockIdx.x == 0 && tid == 0) {
+        atomicExch(a.status, CRC_STEP_BAD_DESCRIPTOR);
+        for (int r = 0; r < a.k; ++r) {
+          a.d_idx[r] = -1;
+          if (a.d_score) a.d_score[r] = __longlong_as_double(0x7ff0000000000000LL);
+        }
+        *a.d_count = 0;
+      }
+      return;
+    }
+    count = n + 1;
+    ext_first = a.step->ext_first;
+    cur = reinterpret_cast<const double*>(a.step->frames);
+  }
   if (tid == 0) {
     double c[3], v[3];
-    chunk_summary(&a.cur.rec[0][0], a.cur.F, c, v);
+    chunk_summary(cur, a.cur.F, c, v);
     for (int e = 0; e < 3; ++e) {
       sh_cn[e] = c[e];
       sh_vn[e] = v[e];
@@ -175,10 +195,10 @@ __global__ void __launch_bounds__(kTopkThreads) retrieve_topk_kernel(const __gri
   List L;
   L.clear();
   const int stride = gridDim.x * blockDim.x;
-  for (int j = blockIdx.x * blockDim.x + tid; j < a.count; j += stride) {
+  for (int j = blockIdx.x * blockDim.x + tid; j < count; j += stride) {
     double s, dist, dot;
     score_entry(a.centre, a.view, j, cn, vn, a.E, a.w_v, s, dist, dot);
-    bool adm = (dist <= a.tau_c) && (dot >= a.cos_tau_v) && (a.n - j >= a.delta) && !(a.exclude_sink && j == 0);
+    bool adm = (dist <= a.tau_c) && (dot >= a.cos_tau_v) && (n - j >= a.delta) && !(a.exclude_sink && j == 0);
     if (adm && a.slab_chunk) adm = a.slab_chunk[j % a.num_slabs] == j;  // its K/V slab still holds it
     if (adm) L.insert(score_key(s), j);
   }
@@ -207,8 +227,9 @@ __global__ void __launch_bounds__(kTopkThreads) retrieve_topk_kernel(const __gri
   }
 
   if (tid == 0) {
-    int count = 0;
-    while (count < a.k && res_j[count] != INT_MAX) ++count;
+    int found = 0;
+    while (found < a.k && res_j[found] != INT_MAX) ++found;
+    const int count = found;
     for (int r = 0; r < a.k; ++r) {
       int chunk;
       double score;
@@ -217,8 +238,8 @@ __global__ void __launch_bounds__(kTopkThreads) retrieve_topk_kernel(const __gri
         score = key_score(res_key[r]);
       } else {
         // the slot extends the recent window with the next-older chunk, if it is kept
-        const int e = a.ext_first - (r - count);
-        const bool ok = a.ext_first >= 0 && e >= a.ext_min &&
+        const int e = ext_first - (r - count);
+        const bool ok = ext_first >= 0 && e >= a.ext_min && e >= 0 &&
                         (a.slab_chunk == nullptr || a.slab_chunk[e % a.num_slabs] == e);
         chunk = ok ? e : -1;
         score = __longlong_as_double(0x7ff0000000000000LL);  // +inf
@@ -239,7 +260,7 @@ __global__ void __launch_bounds__(256, ROPE ? 2 : 4) gather_kernel(const __grid_
   asm volatile("griddepcontrol.wait;" ::: "memory");
   if (threadIdx.x < a.k) plan.chunk[threadIdx.x] = a.d_idx[threadIdx.x];
   __syncthreads();
-  if (ROPE) plan_rope(a.g, a.k, plan);
+  if (ROPE) plan_rope(a.g, a.k, plan, a.g.step ? a.g.step->rope_pos_slot0 : a.g.rope_pos_slot0);
   gather_slots<ROPE>(a.g, a.k, plan);
 }
 

@@ -26,13 +26,14 @@ cache region each chunk occupies and which segments are live at step n.
 
 from __future__ import annotations
 
+import ctypes as C
 import dataclasses
 from typing import List, Optional, Tuple
 
 import numpy as np
 import torch
 
-from . import api
+from . import _abi, api
 
 
 @dataclasses.dataclass
@@ -159,25 +160,126 @@ class ChunkStream:
         return e if e >= 1 else -1
 
     # ---- one chunk step ---------------------------------------------------
+    def window_slot_offset(self, n: int) -> int:
+        """Cache offset that receives chunk n: the sink for chunk 0, else ring slot n % W."""
+        return 0 if n == 0 else self.window_offset(n % self.cfg.window)
+
     def step(self, n: int, frames: np.ndarray, depth: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
              q: torch.Tensor, o: torch.Tensor, lse: Optional[torch.Tensor] = None, stream=None,
-             k_ctl: Optional[torch.Tensor] = None, v_ctl: Optional[torch.Tensor] = None) -> None:
+             k_ctl: Optional[torch.Tensor] = None, v_ctl: Optional[torch.Tensor] = None, events=None) -> None:
+        """One chunk step through the separate entry points.  `events` (five CUDA events)
+        are recorded on `stream` around the update, the retrieval (with the control
+        mirror), the reprojection and the attention, for per-stage timing."""
         c = self.cfg
-        woff = 0 if n == 0 else self.window_offset(n % c.window)
+        s = stream if stream is not None else torch.cuda.current_stream()
+        woff = self.window_slot_offset(n)
         self.cache.segments = self.segments(n)
-        api.crc_cache_update(self.bank, self.shape, n, frames, depth, k_new, v_new, self.cache, woff, stream)
+        if events:
+            events[0].record(s)
+        api.crc_cache_update(self.bank, self.shape, n, frames, depth, k_new, v_new, self.cache, woff, s)
         if self.control_shape is not None:
             self.control_cache.segments = self.cache.segments
             api.crc_cache_update(self.control_bank, self.control_shape, n, frames, depth, k_ctl, v_ctl,
-                                 self.control_cache, woff, stream)
+                                 self.control_cache, woff, s)
+        if events:
+            events[1].record(s)
         params = api.retrieval_params(c.E, c.w_v, c.tau_c, c.cos_tau_v, c.delta, c.k, self.ext_first(n), 1)
         rope = self.rope(n)
         api.crc_retrieve(self.bank, n + 1, self.shape, frames, n, params, self.cache, self.idx, self.score,
-                         self.count, stream, rope=rope)
+                         self.count, s, rope=rope)
         if self.control_shape is not None:
             api.crc_gather(self.control_shape, self.control_bank.kv, self.idx, c.k, self.control_cache, rope=rope,
-                           stream=stream)
+                           stream=s)
+        if events:
+            events[2].record(s)
         api.crc_correspond(self.shape, frames, depth, self.bank, self.idx, self.count, c.k, c.eps, self.uv,
-                           self.cell, self.valid, stream)
+                           self.cell, self.valid, s)
+        if events:
+            events[3].record(s)
         api.crc_biased_attention(self.shape, q, self.cache, o, lse, self.uv, self.valid, c.k, self.idx, c.lam,
-                                 c.sigma, 0, self.status, stream)
+                                 c.sigma, 0, self.status, s)
+        if events:
+            events[4].record(s)
+
+    # ---- the step as one replayed CUDA graph ------------------------------
+    def descriptor(self, n: int, frames: np.ndarray) -> _abi.crc_step:
+        """The per-step values of step n (crc_step): the chunk, its window slot, the
+        fallback chunk, the re-positioning target, the live segments and the frames."""
+        c = self.cfg
+        d = _abi.crc_step()
+        d.n = n
+        d.window_offset = self.window_slot_offset(n)
+        d.ext_first = self.ext_first(n)
+        rope = self.rope(n)
+        d.rope_pos_slot0 = rope.pos_slot0 if rope is not None else 0
+        for g, seg in enumerate(self.segments(n)):
+            d.seg_length[g] = seg[1]
+        rec = np.ascontiguousarray(frames, dtype=np.float64).reshape(-1, 21)
+        if rec.shape[0] != c.F:
+            raise ValueError(f"expected {c.F} frame records")
+        C.memmove(C.addressof(d.frames), rec.ctypes.data, rec.nbytes)
+        return d
+
+    def plan(self, depth: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, q: torch.Tensor, o: torch.Tensor,
+             lse: Optional[torch.Tensor] = None) -> _abi.crc_step_plan:
+        """The fixed part of crc_chunk_step: this stream's bank, cache and outputs, and the
+        input buffers that every step reads (their addresses are captured)."""
+        c = self.cfg
+        if self.control_shape is not None:
+            raise ValueError("the graph-replayed step has no control-branch mirror")
+        p = _abi.crc_step_plan()
+        p.shape = self.shape
+        p.bank = self.bank.struct()
+        full = api.Cache(self.cache.k, self.cache.v, self.segments(c.window + 1))  # every segment at its length
+        p.cache = full.struct()
+        p.retrieval = api.retrieval_params(c.E, c.w_v, c.tau_c, c.cos_tau_v, c.delta, c.k, -1, 1)
+        r = self.rope(c.window + 1)
+        if r is not None:
+            p.rope = r
+        p.eps, p.lam, p.sigma, p.attn_flags = c.eps, c.lam, c.sigma, 0
+        p.d_depth, p.d_k, p.d_v = depth.data_ptr(), k_new.data_ptr(), v_new.data_ptr()
+        p.q, p.o = api.tensor_view(q), api.tensor_view(o)
+        p.d_lse = lse.data_ptr() if lse is not None else None
+        p.d_idx, p.d_score, p.d_count = self.idx.data_ptr(), self.score.data_ptr(), self.count.data_ptr()
+        p.d_uv, p.d_cell, p.d_valid = self.uv.data_ptr(), self.cell.data_ptr(), self.valid.data_ptr()
+        p.d_status = self.status.data_ptr()
+        ws = self.bank.workspace
+        p.d_workspace = ws.data_ptr() if ws is not None else None
+        p.workspace_bytes = 0 if ws is None else ws.numel()
+        return p
+
+    def capture(self, depth: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, q: torch.Tensor,
+                o: torch.Tensor, lse: Optional[torch.Tensor] = None, ring: int = 3) -> None:
+        """Capture one CUDA graph of crc_chunk_step per descriptor slot (`ring` slots, each a
+        device crc_step fed from its own pinned host copy).  replay() then serves every step:
+        the caller fills depth / k_new / v_new / q (the captured buffers) and calls
+        replay(n, frames)."""
+        nb = C.sizeof(_abi.crc_step)
+        self._plan = self.plan(depth, k_new, v_new, q, o, lse)
+        self._h_desc = [torch.zeros(nb, dtype=torch.uint8, pin_memory=True) for _ in range(ring)]
+        self._d_desc = [torch.zeros(nb, dtype=torch.uint8, device=self.idx.device) for _ in range(ring)]
+        self._done = [torch.cuda.Event() for _ in range(ring)]
+        self._graphs = []
+        torch.cuda.synchronize()
+        for i in range(ring):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                api.crc_chunk_step(self._plan, self._d_desc[i], torch.cuda.current_stream())
+            self._graphs.append(g)
+        self._replays = 0
+
+    def replay(self, n: int, frames: np.ndarray, stream=None) -> None:
+        """Step n by graph replay (after capture()): the descriptor goes to the device with one
+        copy on `stream`, then the graph runs.  The host waits only for the step that last used
+        this descriptor slot, `ring` steps ago, before it rewrites the slot's pinned copy."""
+        i = self._replays % len(self._graphs)
+        self._done[i].synchronize()
+        d = self.descriptor(n, frames)
+        C.memmove(self._h_desc[i].data_ptr(), C.addressof(d), C.sizeof(d))
+        s = stream if stream is not None else torch.cuda.current_stream()
+        with torch.cuda.stream(s):
+            self._d_desc[i].copy_(self._h_desc[i], non_blocking=True)
+            self._graphs[i].replay()
+        self._done[i].record(s)
+        self._replays += 1
+        self.cache.segments = self.segments(n)

@@ -59,6 +59,10 @@ _LAYOUT_C = r"""
 #define O(T, f) printf(#T "." #f " %zu\n", offsetof(T, f));
 int main(void) {
   P(crc_frame) P(crc_shape) P(crc_tensor) P(crc_segment) P(crc_cache) P(crc_bank) P(crc_retrieval) P(crc_rope)
+  P(crc_step) P(crc_step_plan) O(crc_step, seg_length) O(crc_step, frames) O(crc_step_plan, bank)
+  O(crc_step_plan, cache) O(crc_step_plan, retrieval) O(crc_step_plan, rope) O(crc_step_plan, eps)
+  O(crc_step_plan, attn_flags) O(crc_step_plan, q) O(crc_step_plan, o) O(crc_step_plan, d_status)
+  O(crc_step_plan, workspace_bytes)
   O(crc_cache, v) O(crc_cache, n_keys) O(crc_cache, seg) O(crc_bank, frames) O(crc_bank, kv) O(crc_bank, slab_chunk)
   O(crc_retrieval, delta) O(crc_retrieval, ext_min) O(crc_retrieval, exclude_sink) O(crc_shape, dtype)
   O(crc_tensor, stride_head) O(crc_rope, frame_pos0) O(crc_rope, theta)
@@ -85,6 +89,15 @@ def test_ctypes_layout_matches_header():
         "crc_tensor": C.sizeof(_abi.crc_tensor), "crc_segment": C.sizeof(_abi.crc_segment),
         "crc_cache": C.sizeof(_abi.crc_cache), "crc_bank": C.sizeof(_abi.crc_bank),
         "crc_retrieval": C.sizeof(_abi.crc_retrieval), "crc_rope": C.sizeof(_abi.crc_rope),
+        "crc_step": C.sizeof(_abi.crc_step), "crc_step_plan": C.sizeof(_abi.crc_step_plan),
+        "crc_step.seg_length": _abi.crc_step.seg_length.offset, "crc_step.frames": _abi.crc_step.frames.offset,
+        "crc_step_plan.bank": _abi.crc_step_plan.bank.offset, "crc_step_plan.cache": _abi.crc_step_plan.cache.offset,
+        "crc_step_plan.retrieval": _abi.crc_step_plan.retrieval.offset,
+        "crc_step_plan.rope": _abi.crc_step_plan.rope.offset, "crc_step_plan.eps": _abi.crc_step_plan.eps.offset,
+        "crc_step_plan.attn_flags": _abi.crc_step_plan.attn_flags.offset,
+        "crc_step_plan.q": _abi.crc_step_plan.q.offset, "crc_step_plan.o": _abi.crc_step_plan.o.offset,
+        "crc_step_plan.d_status": _abi.crc_step_plan.d_status.offset,
+        "crc_step_plan.workspace_bytes": _abi.crc_step_plan.workspace_bytes.offset,
         "crc_retrieval.exclude_sink": _abi.crc_retrieval.exclude_sink.offset,
         "crc_rope.frame_pos0": _abi.crc_rope.frame_pos0.offset, "crc_rope.theta": _abi.crc_rope.theta.offset,
         "crc_cache.v": _abi.crc_cache.v.offset, "crc_cache.n_keys": _abi.crc_cache.n_keys.offset,

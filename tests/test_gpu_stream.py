@@ -254,3 +254,63 @@ def test_stream_resumes_from_a_checkpoint_bit_for_bit(tmp_path):
         assert torch.equal(torch.nan_to_num(u0, nan=-9.0), torch.nan_to_num(u1, nan=-9.0))
     with pytest.raises(ValueError):
         b.load_state_dict({"cache.k": b.cache.k})
+
+
+def test_graph_replayed_stream_matches_the_eager_stream_bit_for_bit():
+    """The 200-step loop-closure stream (2 layers, 2 heads, k = 2, re-positioned keys, 200
+    tracked K/V slabs, a bank of 600 so that the scoring runs on two blocks) through
+    crc_chunk_step replayed from CUDA graphs, against the same stream through the separate
+    entry points: every step's indices, count, scores, correspondences (raw bits, NaN
+    included), cells, flags, output and LSE are identical.  A descriptor whose chunk lies
+    outside the bank is then rejected on the device with CRC_STEP_BAD_DESCRIPTOR."""
+    from paper_2607_21848_gb300 import _abi
+
+    wl = synth.make_workload(5)
+    cfg = crs.StreamConfig(L=2, H=2, d=wl.d, F=wl.F, h=wl.h, w=wl.w, k=wl.k, window=2, capacity=600, num_slabs=200,
+                           E=wl.E, w_v=wl.w_v, tau_c=wl.tau_c, cos_tau_v=wl.cos_tau_v, delta=wl.delta, lam=wl.lam,
+                           sigma=wl.sigma, eps=wl.eps, rope_pairs=22)
+    eager, graph = crs.ChunkStream(cfg), crs.ChunkStream(cfg)
+    assert graph.bank.workspace is not None  # 600 entries: the scoring's blocks meet in the workspace
+    Nc = cfg.Nc
+    g = torch.Generator(device="cuda").manual_seed(21)
+
+    def rnd():
+        return (torch.randn(cfg.L, Nc, cfg.H, cfg.d, generator=g, device="cuda") * wl.qkv_scale).bfloat16()
+
+    kv = [(rnd(), rnd()) for _ in range(5)]
+    q = rnd()
+    o_e, o_g = torch.empty_like(q), torch.empty_like(q)
+    lse_e = torch.empty(cfg.L, cfg.H, Nc, device="cuda")
+    lse_g = torch.empty_like(lse_e)
+    depth_buf = torch.empty(cfg.F, cfg.h, cfg.w, device="cuda")
+    k_buf, v_buf = torch.empty_like(q), torch.empty_like(q)
+    graph.capture(depth_buf, k_buf, v_buf, q, o_g, lse_g)
+    bits = lambda t: t.view(torch.int32)  # noqa: E731
+    closed = 0
+    for n in range(wl.bank_size):
+        fr = synth.frame_records(wl.bank_frames[n])
+        dep = torch.from_numpy(wl.depth_of(n)).cuda()
+        kn, vn = kv[n % 5]
+        eager.step(n, fr, dep, kn, vn, q, o_e, lse_e)
+        depth_buf.copy_(dep)
+        k_buf.copy_(kn)
+        v_buf.copy_(vn)
+        graph.replay(n, fr)
+        torch.cuda.synchronize()
+        assert eager.status.item() == 0 and graph.status.item() == 0, n
+        assert torch.equal(eager.idx, graph.idx) and torch.equal(eager.count, graph.count), n
+        assert torch.equal(eager.score, graph.score), n
+        assert torch.equal(bits(eager.uv), bits(graph.uv)), n
+        assert torch.equal(eager.cell, graph.cell) and torch.equal(eager.valid, graph.valid), n
+        assert torch.equal(o_e, o_g), n
+        assert torch.equal(bits(lse_e), bits(lse_g)), n
+        closed += int(graph.count.item()) > 0
+    assert closed >= 40  # the loop closes after one lap: retrieved chunks go through the replayed step
+    assert torch.equal(eager.bank.frames, graph.bank.frames) and torch.equal(eager.cache.k, graph.cache.k)
+    # chunk 600 is outside a bank of 600: nothing is written, the status word says why
+    frames_before = graph.bank.frames.clone()
+    graph.replay(600, synth.frame_records(wl.bank_frames[0]))
+    torch.cuda.synchronize()
+    assert graph.status.item() == _abi.CRC_STEP_BAD_DESCRIPTOR
+    assert int(graph.count.item()) == 0 and bool((graph.idx < 0).all())
+    assert torch.equal(graph.bank.frames, frames_before)
