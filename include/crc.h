@@ -50,6 +50,7 @@ typedef int32_t crc_status;
 #define CRC_ERR_UNSUPPORTED 3  /* dtype / head dim / alignment / device not handled */
 #define CRC_ERR_CUDA 4         /* a CUDA call failed; see crc_last_cuda_error()     */
 #define CRC_ERR_DEVICE 5       /* a kernel reported a failure in its status word    */
+#define CRC_ERR_TOO_LARGE 6    /* beyond the fixed scratch of crc_retrieve_noalloc  */
 
 /* ---- element types ------------------------------------------------------- */
 #define CRC_F32 0
@@ -263,6 +264,35 @@ crc_status crc_retrieve(const crc_bank* bank, int32_t bank_count, const crc_shap
  * slots: 0 up to 512 entries, else 16 bytes per (block of 512 entries, slot) plus
  * 256, rounded up (under 300 KB for any bank).  0 for invalid arguments. */
 size_t crc_retrieve_workspace_size(int32_t bank_count, int32_t k);
+
+/*
+ * crc_retrieve_noalloc — crc_retrieve for callers that cannot allocate device memory.
+ * (The paper has no counterpart: this is a deployment variant of the same call.)
+ *
+ * Who needs it: an engine's render thread with a fixed per-frame budget (cudaMalloc
+ * and cudaFree can synchronise the device and take milliseconds), a plugin whose host
+ * application owns all GPU memory, or a stream that must not fail half-way with an
+ * out-of-memory error.  Instead of a caller workspace, banks of more than 512 entries
+ * use a fixed scratch array inside the library's device code, CRC_NOALLOC_SCRATCH_BYTES
+ * (64 KiB) on every GPU that loads the library, held until the process exits.  Nothing
+ * is allocated or freed by the call.
+ *
+ * Arguments, results and errors are those of crc_retrieve, plus CRC_ERR_TOO_LARGE when
+ * crc_retrieve_workspace_size(bank_count, k) exceeds the scratch (at k = 8 that is a
+ * bank of more than 261 120 entries; at k = 1 no bank is too large), and CRC_ERR_CUDA
+ * when the scratch's device address cannot be found.
+ * The first call on each device that needs the scratch looks up its device address
+ * (cudaGetSymbolAddress, once per device, with that device current); make that first
+ * call before capturing any stream on that device.  Every call shares the one array,
+ * which keeps the previous call's contents (each call clears what must start at zero):
+ * calls that may overlap on the GPU -- on different streams, or from different host
+ * threads -- race on it, so they must be ordered, e.g. on one stream.
+ */
+#define CRC_NOALLOC_SCRATCH_BYTES 65536
+crc_status crc_retrieve_noalloc(const crc_bank* bank, int32_t bank_count, const crc_shape* shape,
+                                const crc_frame* cur, int32_t n, const crc_retrieval* p, const crc_cache* cache,
+                                const crc_rope* rope, int32_t* d_idx, double* d_score, int32_t* d_count,
+                                cudaStream_t s);
 
 /*
  * crc_gather — the gather half of crc_retrieve for a second cache that mirrors

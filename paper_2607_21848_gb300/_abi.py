@@ -17,6 +17,8 @@ CRC_ERR_SHAPE = 2
 CRC_ERR_UNSUPPORTED = 3
 CRC_ERR_CUDA = 4
 CRC_ERR_DEVICE = 5
+CRC_ERR_TOO_LARGE = 6
+CRC_NOALLOC_SCRATCH_BYTES = 65536
 
 CRC_F32 = 0
 CRC_BF16 = 1
@@ -107,6 +109,9 @@ _SIGS = {
                                  _P(crc_retrieval), _P(crc_cache), _P(crc_rope), C.c_void_p, C.c_void_p, C.c_void_p,
                                  C.c_void_p, C.c_size_t, C.c_void_p]),
     "crc_retrieve_workspace_size": (C.c_size_t, [C.c_int32, C.c_int32]),
+    "crc_retrieve_noalloc": (C.c_int32, [_P(crc_bank), C.c_int32, _P(crc_shape), _P(crc_frame), C.c_int32,
+                                         _P(crc_retrieval), _P(crc_cache), _P(crc_rope), C.c_void_p, C.c_void_p,
+                                         C.c_void_p, C.c_void_p]),
     "crc_gather": (C.c_int32, [_P(crc_shape), C.c_void_p, C.c_int32, C.c_void_p, C.c_int32, _P(crc_cache),
                                _P(crc_rope), C.c_void_p]),
     "crc_correspond": (C.c_int32, [_P(crc_shape), _P(crc_frame), C.c_void_p, _P(crc_bank), C.c_void_p, C.c_void_p,

@@ -195,6 +195,23 @@ def crc_retrieve(bank: Bank, bank_count: int, shp: _abi.crc_shape, cur_frames: n
                                 0 if ws is None else ws.numel() * ws.element_size(), _stream(stream)))
 
 
+def crc_retrieve_noalloc(bank: Bank, bank_count: int, shp: _abi.crc_shape, cur_frames: np.ndarray, n: int,
+                         params: _abi.crc_retrieval, cache: Optional[Cache], idx: torch.Tensor,
+                         score: Optional[torch.Tensor], count: torch.Tensor, stream=None,
+                         rope: Optional[_abi.crc_rope] = None) -> None:
+    """crc_retrieve with the library's fixed scratch in place of a workspace, for callers
+    that cannot allocate device memory (see include/crc.h)."""
+    lib = _abi.load()
+    fr = frames_struct(cur_frames)
+    b = bank.struct()
+    cs = cache.struct() if cache is not None else None
+    _abi.check("crc_retrieve_noalloc",
+               lib.crc_retrieve_noalloc(C.byref(b), bank_count, C.byref(shp), fr, n, C.byref(params),
+                                        C.byref(cs) if cs is not None else None,
+                                        C.byref(rope) if rope is not None else None, _ptr(idx), _ptr(score),
+                                        _ptr(count), _stream(stream)))
+
+
 def crc_gather(shp: _abi.crc_shape, pool: torch.Tensor, idx: torch.Tensor, k: int, cache: Cache,
                rope: Optional[_abi.crc_rope] = None, stream=None) -> None:
     """Mirror the retrieved slots d_idx of a step into a second cache from its own slab pool

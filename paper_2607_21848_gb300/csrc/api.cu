@@ -392,6 +392,7 @@ const char* crc_status_string(crc_status st) {
     case CRC_ERR_UNSUPPORTED: return "unsupported dtype, head dim, alignment or device";
     case CRC_ERR_CUDA: return "CUDA error";
     case CRC_ERR_DEVICE: return "kernel reported a failure";
+    case CRC_ERR_TOO_LARGE: return "beyond the fixed scratch of the no-allocation entry point";
     default: return "unknown status";
   }
 }

@@ -47,7 +47,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 def test_version_and_status_strings(lib):
     assert "sm_103a" in lib.crc_version().decode()
-    for st in range(6):
+    for st in range(7):
         assert lib.crc_status_string(st).decode()
 
 
