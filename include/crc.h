@@ -60,6 +60,8 @@ typedef int32_t crc_status;
 #define CRC_SEG_SINK 0       /* the anchor: the first chunk, never evicted          */
 #define CRC_SEG_RETRIEVED 1  /* a pose-retrieved slot; `slot` = retrieval rank r    */
 #define CRC_SEG_WINDOW 2     /* the recent window (including the current chunk)     */
+#define CRC_SEG_CURRENT 3    /* the window slot holding the current chunk (length N_c or 0): a
+                                window segment, except under CRC_ATTN_FRAME_CAUSAL     */
 
 #define CRC_MAX_SEGMENTS 16
 #define CRC_MAX_FRAMES 4   /* frames per chunk, F */
@@ -348,6 +350,9 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
                                 on the tensor-core kernel, which adds the bonus to each biased tile's
                                 scores in the softmax; otherwise the SIMT kernel.  Not combined with
                                 CRC_ATTN_SKIP_FAR, which is then ignored. */
+#define CRC_ATTN_FRAME_CAUSAL 16  /* test mode of the block-causal reading: inside the current chunk
+                                     (its CRC_SEG_CURRENT segment) a query of latent frame t sees
+                                     only the keys of frames <= t; every other key stays visible */
 #define CRC_ATTN_BIAS_DIRECT 8  /* tensor-core kernel, Eq. 2 form: evaluate the bias per score in the
                                    softmax (exact to fp32 rounding) even where the tensor-core
                                    expansion is within its error limit (see crc_biased_attention) */
@@ -367,7 +372,10 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
  *             segment) / (h*w), u_k its (x, y) in that frame, and d_valid[p][s];
  *             0 for every other key (sink, window) and for invalid pairs.
  * Softmax runs over the active keys: keys inside a segment, minus retrieved slots
- * whose chunk is empty (d_slot_chunk[r] < 0, when d_slot_chunk is not NULL).
+ * whose chunk is empty (d_slot_chunk[r] < 0, when d_slot_chunk is not NULL), and, with
+ * CRC_ATTN_FRAME_CAUSAL, minus the current chunk's keys of frames after the query's
+ * (query p lies in frame p / (h w); a key at position i of the CRC_SEG_CURRENT
+ * segment in frame i / (h w)).
  * The bias is evaluated inside the tile loop and never stored.
  *
  *   q         [L][n_q][H][d] queries (dtype of the call); n_q = N_c.

@@ -9,6 +9,7 @@ from .crc_oracle import (  # noqa: F401
     bias_matrix,
     chunk_pose,
     correspond,
+    current_key_frames,
     fill_slots,
     gather,
     key_table,

@@ -46,6 +46,7 @@ import numpy as np
 SEG_SINK = 0
 SEG_RETRIEVED = 1
 SEG_WINDOW = 2
+SEG_CURRENT = 3  # the window slot holding the current chunk (a window segment otherwise)
 
 
 # ----------------------------------------------------------------------------
@@ -305,13 +306,28 @@ def bias_matrix(uv: np.ndarray, valid: np.ndarray, rows: np.ndarray, src: np.nda
     return B
 
 
+def current_key_frames(segments, n_keys: int, h: int, w: int) -> np.ndarray:
+    """Per key column: the latent frame of the current chunk the key belongs to (keys of
+    the CURRENT segment, position // (h w)), -1 for every other key."""
+    kf = np.full(n_keys, -1, dtype=np.int64)
+    for off, length, kind, _ in segments:
+        if kind == SEG_CURRENT and length > 0:
+            kf[off:off + length] = np.arange(length) // (h * w)
+    return kf
+
+
 def attention(Q: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, uv: np.ndarray, valid: np.ndarray,
               segments, h: int, w: int, F: int, lam: float, sigma: float,
               slot_chunks: Optional[np.ndarray] = None, rows: Optional[np.ndarray] = None,
               layers: Optional[Sequence[int]] = None, heads: Optional[Sequence[int]] = None,
-              row_block: int = 1024, bias_form: str = "eq2"):
+              row_block: int = 1024, bias_form: str = "eq2", mask_mode: str = "chunk"):
     """Eq. 2: O_p = sum_k softmax_k(A_pk) V_k with A_pk = q_p.k_k / sqrt(d) + lam B_s(p, k).
     bias_form selects the bias of `bias_matrix` (Eq. 2, or the opt-in additive Gaussian).
+
+    mask_mode "chunk": every active key is visible to every query (chunks attend
+    block-causally, Sec. 3, and every cached key belongs to this chunk or an earlier one).
+    "frame": frame-causal inside the current chunk -- a query of latent frame t = p // (h w)
+    does not see the keys of the CURRENT segment whose frame is later than t.
 
     Q [L, Nq, H, d], Kc/Vc [L, Nk, H, d] (values as given, widened to fp64),
     uv [Nq, S, 2], valid [Nq, S].  Softmax runs over the active keys only, in two
@@ -325,6 +341,9 @@ def attention(Q: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, uv: np.ndarray, val
     heads = list(range(H)) if heads is None else list(heads)
     active, src, ux, uy = key_table(segments, Nk, h, w, F, slot_chunks)
     act = np.nonzero(active)[0]
+    if mask_mode not in ("chunk", "frame"):
+        raise ValueError(mask_mode)
+    kframe = current_key_frames(segments, Nk, h, w)[act]
     O = np.zeros((len(layers), rows.shape[0], len(heads), d))
     lse = np.zeros((len(layers), len(heads), rows.shape[0]))
     scale = 1.0 / math.sqrt(d)
@@ -337,6 +356,9 @@ def attention(Q: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, uv: np.ndarray, val
                 k = Kc[l, act, hh, :].astype(np.float64)
                 v = Vc[l, act, hh, :].astype(np.float64)
                 A = (q @ k.T) * scale + lamB
+                if mask_mode == "frame":
+                    qframe = rb // (h * w)
+                    A = np.where(kframe[None, :] > qframe[:, None], -np.inf, A)
                 m = A.max(axis=1, keepdims=True)
                 e = np.exp(A - m)
                 ssum = e.sum(axis=1, keepdims=True)

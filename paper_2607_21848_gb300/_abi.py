@@ -26,6 +26,7 @@ CRC_BF16 = 1
 CRC_SEG_SINK = 0
 CRC_SEG_RETRIEVED = 1
 CRC_SEG_WINDOW = 2
+CRC_SEG_CURRENT = 3
 
 CRC_MAX_SEGMENTS = 16
 CRC_MAX_FRAMES = 4
@@ -37,6 +38,7 @@ CRC_ATTN_SIMT = 1
 CRC_ATTN_GAUSSIAN = 2
 CRC_ATTN_SKIP_FAR = 4
 CRC_ATTN_BIAS_DIRECT = 8
+CRC_ATTN_FRAME_CAUSAL = 16
 
 
 class crc_frame(C.Structure):

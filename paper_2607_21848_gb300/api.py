@@ -21,11 +21,13 @@ from ._abi import CrcError  # noqa: F401
 SEG_SINK = _abi.CRC_SEG_SINK
 SEG_RETRIEVED = _abi.CRC_SEG_RETRIEVED
 SEG_WINDOW = _abi.CRC_SEG_WINDOW
+SEG_CURRENT = _abi.CRC_SEG_CURRENT
 ATTN_DEFAULT = _abi.CRC_ATTN_DEFAULT
 ATTN_SIMT = _abi.CRC_ATTN_SIMT
 ATTN_GAUSSIAN = _abi.CRC_ATTN_GAUSSIAN
 ATTN_SKIP_FAR = _abi.CRC_ATTN_SKIP_FAR
 ATTN_BIAS_DIRECT = _abi.CRC_ATTN_BIAS_DIRECT
+ATTN_FRAME_CAUSAL = _abi.CRC_ATTN_FRAME_CAUSAL
 
 
 def _dtype_code(dt: torch.dtype) -> int:
@@ -117,6 +119,10 @@ class Cache:
     def n_keys(self) -> int:
         return self.k.shape[1]
 
+    def heads(self, h0: int, count: int) -> "Cache":
+        """The same cache restricted to heads [h0, h0 + count): strided views, same segments."""
+        return Cache(head_view(self.k, h0, count), head_view(self.v, h0, count), self.segments)
+
     def struct(self) -> _abi.crc_cache:
         c = _abi.crc_cache()
         c.k = tensor_view(self.k)
@@ -128,6 +134,22 @@ class Cache:
         for i, (off, length, kind, slot) in enumerate(self.segments):
             c.seg[i] = _abi.crc_segment(off, length, kind, slot)
         return c
+
+
+def head_range(H: int, rank: int, world: int) -> Tuple[int, int]:
+    """Heads [h0, h0 + count) of rank `rank` when H heads are split over `world` ranks as
+    evenly as possible (heads are independent in Eq. 2, so each rank runs its own range
+    with its own bank and cache views; nothing is exchanged)."""
+    if world < 1 or not 0 <= rank < world or H < world:
+        raise ValueError("need 0 <= rank < world <= H")
+    base, extra = divmod(H, world)
+    h0 = rank * base + min(rank, extra)
+    return h0, base + (1 if rank < extra else 0)
+
+
+def head_view(t: torch.Tensor, h0: int, count: int) -> torch.Tensor:
+    """Heads [h0, h0 + count) of a [L, N, H, d] tensor, as a strided view of the same memory."""
+    return t[:, :, h0:h0 + count, :]
 
 
 def retrieval_params(E: float, w_v: float, tau_c: float, cos_tau_v: float, delta: int, k: int,

@@ -82,9 +82,11 @@ crc_status check_cache(const crc_cache* c, const crc_shape* sh) {
   for (int g = 0; g < c->nseg; ++g) {
     const crc_segment& s = c->seg[g];
     if (s.offset < 0 || s.length < 0 || (int64_t)s.offset + s.length > c->n_keys) return CRC_ERR_SHAPE;
-    if (s.kind != CRC_SEG_SINK && s.kind != CRC_SEG_RETRIEVED && s.kind != CRC_SEG_WINDOW) return CRC_ERR_INVALID_ARG;
+    if (s.kind != CRC_SEG_SINK && s.kind != CRC_SEG_RETRIEVED && s.kind != CRC_SEG_WINDOW && s.kind != CRC_SEG_CURRENT)
+      return CRC_ERR_INVALID_ARG;
     if (s.kind == CRC_SEG_RETRIEVED && (s.slot < 0 || s.slot >= CRC_MAX_K || (s.length != 0 && s.length != nc)))
       return CRC_ERR_SHAPE;
+    if (s.kind == CRC_SEG_CURRENT && s.length != 0 && s.length != nc) return CRC_ERR_SHAPE;
     for (int h2 = 0; h2 < g; ++h2) {  // segments may not overlap
       const crc_segment& o = c->seg[h2];
       if (s.length > 0 && o.length > 0 && s.offset < o.offset + o.length && o.offset < s.offset + s.length)
@@ -314,7 +316,7 @@ crc_status prep_attention(crc::AttnArgs& a, bool& tc, const crc_shape* shape, cr
   if (n_q != nc) return CRC_ERR_SHAPE;
   if (k < 0 || k > CRC_MAX_K || !isfinite(lambda) || lambda < 0.f || !(sigma > 0.f) || !isfinite(sigma))
     return CRC_ERR_INVALID_ARG;
-  if (flags & ~(CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN | CRC_ATTN_SKIP_FAR | CRC_ATTN_BIAS_DIRECT))
+  if (flags & ~(CRC_ATTN_SIMT | CRC_ATTN_GAUSSIAN | CRC_ATTN_SKIP_FAR | CRC_ATTN_BIAS_DIRECT | CRC_ATTN_FRAME_CAUSAL))
     return CRC_ERR_INVALID_ARG;
   bool any_ret = false, any_other = false;
   for (int g = 0; g < cache->nseg; ++g) {
@@ -366,6 +368,7 @@ crc_status prep_attention(crc::AttnArgs& a, bool& tc, const crc_shape* shape, cr
   a.status = d_status;
   a.bias_form = (flags & CRC_ATTN_GAUSSIAN) ? 1 : 0;
   a.bias_direct = (flags & CRC_ATTN_BIAS_DIRECT) ? 1 : 0;
+  a.frame_causal = (flags & CRC_ATTN_FRAME_CAUSAL) ? 1 : 0;
   // skipped weights are scaled by at most 2^-64: lambda d^2 / (2 sigma^2) >= 64 ln 2
   a.skip_far = (flags & CRC_ATTN_SKIP_FAR) && !(flags & CRC_ATTN_GAUSSIAN) && lambda > 0.f && any_ret && any_other &&
                        d_valid

@@ -97,6 +97,7 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const __grid_constant__ 
         }
       }
       if (!ki.active) logit = -INFINITY;
+      if (a.frame_causal && ki.frame > p / (a.h * a.w)) logit = -INFINITY;  // a later frame of this chunk
       float tmax = logit;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));

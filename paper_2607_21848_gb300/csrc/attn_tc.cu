@@ -137,7 +137,7 @@ struct TileInfo {
   uint8_t nact_m1;  // active keys - 1 (keys key0 .. key0 + nact - 1)
   uint8_t cls;
   int8_t s;         // source frame of the (biased) keys, -1 for an unbiased tile
-  uint8_t pad;
+  uint8_t kf1;      // current-chunk tiles: 1 + the keys' frame (frame-causal mask), else 0
   uint16_t q;       // ordinal among CLS_AUG tiles (ring position)
   uint16_t loc0;    // index of key0 inside its source frame (biased tiles)
 };
@@ -356,11 +356,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int len = seg_length(a, g);
       if (len <= 0) continue;
       const bool ret = sg.kind == CRC_SEG_RETRIEVED;
+      // the current chunk's segment is cut per frame too when the frame-causal mask is on
+      const bool curc = sg.kind == CRC_SEG_CURRENT && a.frame_causal;
       if (ret && a.slot_chunk && a.slot_chunk[sg.slot] < 0) continue;  // empty slot: masked
-      const int nr = ret ? a.F : 1;
+      const int nr = (ret || curc) ? a.F : 1;
       for (int rr = 0; rr < nr; ++rr) {
-        const int rstart = ret ? sg.offset + rr * hw : sg.offset;
-        const int rlen = ret ? hw : len;
+        const int rstart = (ret || curc) ? sg.offset + rr * hw : sg.offset;
+        const int rlen = (ret || curc) ? hw : len;
         const int ntile = (rlen + BN - 1) / BN;
         for (int base = 0; base < ntile; base += 32) {
           const int t = base + lane;
@@ -371,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ti.nact_m1 = (uint8_t)(nact - 1);
           ti.s = ret ? (int8_t)(sg.slot * a.F + rr) : (int8_t)-1;
           ti.cls = (nact == BN && !ret) ? CLS_PLAIN : CLS_AUG;
-          ti.pad = 0;
+          ti.kf1 = curc ? (uint8_t)(rr + 1) : 0;
           ti.loc0 = (uint16_t)(t * BN);
           bool keep = act;
           if (skip_far && ret && act) {
@@ -636,6 +638,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int p = q0 + x * BM + r;    // query index
     if (q0 + x * BM < a.Nq) {         // else: a query tile without any query, no MMA runs for it
     const bool row_ok = p < a.Nq;
+    const int qframe = p / (a.h * a.w);  // the query's latent frame (frame-causal mode)
     const uint32_t trow = tmem + ((uint32_t)(wq * 32) << 16);
     const uint32_t tS = trow + TM_S + 128u * x;
     const uint32_t tO = trow + TM_O + 128u * x;
@@ -715,6 +718,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
+      // frame-causal mode: a tile of the current chunk's frame f is invisible to this row when
+      // the row's query frame is earlier; its weights are then 2^-inf = 0 and m, l stay put
+      bool rowmask = false;
+      if (a.frame_causal) {
+        const int kf1 = tiles[j].kf1;
+        rowmask = kf1 > 0 && kf1 - 1 > qframe;
+      }
       // row max: eight running three-input max chains, then a final fold
       float mx[8];
 #pragma unroll
@@ -723,13 +733,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c = 16; c < 128; c += 16)
 #pragma unroll
         for (int i = 0; i < 8; ++i) mx[i] = max3f(mx[i], __uint_as_float(sr[c + i]), __uint_as_float(sr[c + 8 + i]));
-      const float mt = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sc;
+      const float mt = rowmask ? -INFINITY
+                               : max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sc;
       // base-2 online softmax; the max is refreshed only when it grows by > 8
       const float mnew = fmaxf(m, mt);
       const bool resc = mnew > m + 8.f;
       const float factor = resc ? ex2(m - mnew) : 1.f;
       if (resc) m = mnew;
-      const uint64_t NM2 = pk2(-m, -m);
+      const uint64_t NM2 = rowmask ? pk2(-INFINITY, -INFINITY) : pk2(-m, -m);
       uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
@@ -860,7 +871,7 @@ bool attn_tc_supported(const AttnArgs& a) {
   for (int g = 0; g < a.nseg; ++g) {
     const crc_segment& sg = a.seg[g];
     if (sg.length <= 0) continue;
-    if (sg.kind == CRC_SEG_RETRIEVED)
+    if (sg.kind == CRC_SEG_RETRIEVED || (sg.kind == CRC_SEG_CURRENT && a.frame_causal))
       ntiles += (int64_t)a.F * ((a.h * a.w + BN - 1) / BN);
     else
       ntiles += (sg.length + BN - 1) / BN;

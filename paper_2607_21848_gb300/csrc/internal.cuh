@@ -198,16 +198,17 @@ struct AttnArgs {
   int32_t* status;
   int32_t bias_form;  // 0: Eq. 2 quadratic; 1: additive Gaussian (CRC_ATTN_GAUSSIAN)
   int32_t bias_direct;  // Eq. 2 evaluated per score even where the tensor-core expansion is accurate
+  int32_t frame_causal; // CRC_ATTN_FRAME_CAUSAL: later frames of the CURRENT segment are masked per query
   int32_t skip_far;   // CRC_ATTN_SKIP_FAR in force (tensor-core kernel)
   float skip_d2;      // squared grid distance beyond which a retrieved tile is skipped
 };
 // Length of cache segment g in this call: the descriptor's, clamped to the plan's.
-// A retrieved segment is all or nothing (N_c keys or none).
+// A retrieved or current-chunk segment is all or nothing (N_c keys or none).
 __device__ __forceinline__ int32_t seg_length(const AttnArgs& a, int g) {
   const int32_t len = a.seg[g].length;
   if (a.step == nullptr) return len;
   const int32_t sl = a.step->seg_length[g];
-  if (a.seg[g].kind == CRC_SEG_RETRIEVED) return sl > 0 ? len : 0;
+  if (a.seg[g].kind == CRC_SEG_RETRIEVED || a.seg[g].kind == CRC_SEG_CURRENT) return sl > 0 ? len : 0;
   return sl < 0 ? 0 : (sl < len ? sl : len);
 }
 

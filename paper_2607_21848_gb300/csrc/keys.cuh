@@ -10,12 +10,13 @@ namespace crc {
 
 struct KeyInfo {
   int active;
-  int src;  // -1: no bias on this column
+  int src;    // -1: no bias on this column
+  int frame;  // keys of the current chunk (CRC_SEG_CURRENT): their latent frame, else -1
   float x, y;
 };
 
 __device__ __forceinline__ KeyInfo key_info_of(const AttnArgs& a, int key) {
-  KeyInfo ki{0, -1, 0.f, 0.f};
+  KeyInfo ki{0, -1, -1, 0.f, 0.f};
   if (key >= a.Nk) return ki;
   for (int g = 0; g < a.nseg; ++g) {
     const crc_segment sg = a.seg[g];
@@ -30,6 +31,8 @@ __device__ __forceinline__ KeyInfo key_info_of(const AttnArgs& a, int key) {
       ki.src = sg.slot * a.F + fr;
       ki.y = (float)row;
       ki.x = (float)(rem - row * a.w);
+    } else if (sg.kind == CRC_SEG_CURRENT) {
+      ki.frame = (key - sg.offset) / (a.h * a.w);
     }
     ki.active = 1;
     return ki;

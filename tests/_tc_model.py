@@ -87,32 +87,37 @@ def exact_bias_raw(ux, uy, xk, yk, lam, sigma, d: int = 128):
     return -lam * math.sqrt(d) * d2 / (2.0 * sigma * sigma)
 
 
-def kernel_tiles(segments, h, w, F, slot_chunks=None, BN=128):
+def kernel_tiles(segments, h, w, F, slot_chunks=None, BN=128, frame_causal=False):
     """The kernel's KV tiles: (first key, active keys, source frame or -1, index of the
-    first key inside its frame), in segment order, retrieved segments cut per frame."""
+    first key inside its frame, current-chunk frame or -1), in segment order, retrieved
+    segments (and, in the frame-causal mode, the current chunk's) cut per frame."""
     tiles = []
     hw = h * w
     for off, length, kind, slot in segments:
         if length <= 0:
             continue
-        ret = kind == 1
+        ret, cur = kind == 1, kind == 3 and frame_causal
         if ret and slot_chunks is not None and slot_chunks[slot] < 0:
             continue
-        for rr in range(F if ret else 1):
-            start = off + rr * hw if ret else off
-            rlen = hw if ret else length
+        for rr in range(F if (ret or cur) else 1):
+            start = off + rr * hw if (ret or cur) else off
+            rlen = hw if (ret or cur) else length
             for t in range((rlen + BN - 1) // BN):
-                tiles.append((start + t * BN, min(BN, rlen - t * BN), slot * F + rr if ret else -1, t * BN))
+                tiles.append((start + t * BN, min(BN, rlen - t * BN), slot * F + rr if ret else -1, t * BN,
+                              rr if cur else -1))
     return tiles
 
 
-def attention_model(Q, Kc, Vc, uv, valid, segments, h, w, F, lam, sigma, slot_chunks=None, bias="tensor"):
+def attention_model(Q, Kc, Vc, uv, valid, segments, h, w, F, lam, sigma, slot_chunks=None, bias="tensor",
+                    mask_mode="chunk"):
     """O [L, Nq, H, d] (bf16 values as float64) and LSE [L, H, Nq] following the kernel's
     rounding steps.  bias = "tensor" (the K = 16 expansion, exact products) or "direct"
-    (fp32 per score, as the kernel's per-score form)."""
+    (fp32 per score, as the kernel's per-score form).  mask_mode = "frame": a row whose
+    query frame precedes a current-chunk tile's frame takes no weight from that tile and
+    keeps its max and sum."""
     L, Nq, H, d = Q.shape
     sc, coef, inv_sc = kernel_constants(lam, sigma, d)
-    tiles = kernel_tiles(segments, h, w, F, slot_chunks)
+    tiles = kernel_tiles(segments, h, w, F, slot_chunks, frame_causal=mask_mode == "frame")
     O = np.zeros((L, Nq, H, d))
     LSE = np.zeros((L, H, Nq))
     uv32 = np.asarray(uv, np.float32)
@@ -122,7 +127,9 @@ def attention_model(Q, Kc, Vc, uv, valid, segments, h, w, F, lam, sigma, slot_ch
             m = np.full(Nq, -np.inf, np.float32)
             lsum = np.zeros(Nq, np.float32)
             acc = np.zeros((Nq, d), np.float32)
-            for j, (k0, nact, s, loc0) in enumerate(tiles):
+            qframe = np.arange(Nq) // (h * w)
+            for j, (k0, nact, s, loc0, kf) in enumerate(tiles):
+                rowmask = (kf >= 0) & (kf > qframe)
                 kk = Kc[l, k0:k0 + nact, hh, :].astype(np.float64)
                 vv = Vc[l, k0:k0 + nact, hh, :].astype(np.float64)
                 S = q @ kk.T  # exact products; fp32 rounding below
@@ -140,13 +147,14 @@ def attention_model(Q, Kc, Vc, uv, valid, segments, h, w, F, lam, sigma, slot_ch
                         b = (araw * d2.astype(np.float64))
                     S = S + np.where(ok[:, None], b, 0.0)
                 S32 = S.astype(np.float32)
-                mt = (S32.max(axis=1) * sc).astype(np.float32)
+                mt = np.where(rowmask, -np.inf, (S32.max(axis=1) * sc)).astype(np.float32)
                 mnew = np.maximum(m, mt)
                 resc = mnew > (m + f32(8.0)).astype(np.float32)
                 with np.errstate(invalid="ignore", over="ignore"):
                     factor = np.where(resc, np.exp2((m - mnew).astype(np.float64)).astype(np.float32), f32(1.0))
                 m = np.where(resc, mnew, m).astype(np.float32)
                 t = (S32.astype(np.float64) * float(sc) - m[:, None].astype(np.float64)).astype(np.float32)
+                t[rowmask] = -np.inf
                 p = np.exp2(t.astype(np.float64)).astype(np.float32)
                 psum = p.astype(np.float64).sum(axis=1).astype(np.float32)
                 lsum = (lsum * factor + psum).astype(np.float32)

@@ -262,7 +262,7 @@ def test_attention_rejects_bad_parameters(lib):
     assert _attend(lib, sigma=math.inf) == INVALID
     assert _attend(lib, k=-1) == INVALID
     assert _attend(lib, k=_abi.CRC_MAX_K + 1) == INVALID
-    assert _attend(lib, flags=16) == INVALID            # unknown flag bit
+    assert _attend(lib, flags=32) == INVALID            # unknown flag bit
     assert _attend(lib, uv=None) == INVALID             # retrieved segments need correspondences
     assert _attend(lib, valid=None) == INVALID
     assert _attend(lib, k=0) == SHAPE                   # a retrieved segment's slot must be < k
@@ -281,6 +281,8 @@ def test_attention_rejects_bad_segment_tables(lib):
     assert _attend(lib, cache=too_many) == SHAPE
     misaligned = _cache(k_data=_ptr(6) + 8)
     assert _attend(lib, cache=misaligned) == UNSUPPORTED
+    # the current chunk's segment is a whole chunk (cut per frame), or empty
+    assert _attend(lib, cache=_cache([(0, NC - 1, _abi.CRC_SEG_CURRENT, 0)], NC)) == SHAPE
 
 
 def test_attention_limits_of_the_tensor_core_kernel(lib):

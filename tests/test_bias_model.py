@@ -93,6 +93,7 @@ def test_kernel_tiles_cut_segments_and_retrieved_frames():
     # sink: 37 tiles (36 full + 72 keys); retrieved: 3 frames x 13 tiles (12 full + 24 keys); window: 74 tiles
     assert len(tiles) == 37 + 39 + 74
     ret = [t for t in tiles if t[2] >= 0]
+    assert all(t[4] == -1 for t in tiles)  # no current-chunk segment here
     assert [t[2] for t in ret] == [0] * 13 + [1] * 13 + [2] * 13
     assert ret[12][1] == 1560 - 12 * 128 and ret[13][0] == 4680 + 1560 and ret[13][3] == 0
     assert sum(t[1] for t in tiles) == 4680 + 4680 + 9360

@@ -94,7 +94,8 @@ def _ulp_bf16(x):
     return 2.0 ** (np.floor(np.log2(a)) - 7)
 
 
-def _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, lam, sigma, bias="tensor"):
+def _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, lam, sigma, bias="tensor",
+                                     mask_mode="chunk"):
     """The tensor-core output against a CPU model of the kernel's own rounding steps
     (tests/_tc_model.py: tiles cut per segment and frame, the stale row max, P rounded to
     bf16 at the kernel's scale, the expansion's coefficients as the kernel rounds them).
@@ -107,8 +108,8 @@ def _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, l
     from tests import _tc_model as model
 
     F, h, w, k = geom
-    Om, _ = model.attention_model(Q, Kc, Vc, uv, valid, segs, h, w, F, lam, sigma, bias=bias)
-    Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, lam, sigma)
+    Om, _ = model.attention_model(Q, Kc, Vc, uv, valid, segs, h, w, F, lam, sigma, bias=bias, mask_mode=mask_mode)
+    Oabs, _ = _oracle(Q, Kc, np.abs(Vc), uv, valid, segs, geom, lam, sigma, mask_mode=mask_mode)
     dm = np.abs(Og - Om)
     slack = _ulp_bf16(Om) + 2.0 ** -9 * Oabs
     assert (dm == 0).mean() >= 0.99, (dm == 0).mean()
@@ -380,6 +381,68 @@ def test_bf16_direct_form_follows_the_kernel_model_on_32_source_frames():
     _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, 4.0, 1.0, bias="direct")
 
 
+# ---------------------------------------------------------------------------- frame-causal test mode
+def _with_current(segs):
+    """The same segments with the last window slot marked as the current chunk's."""
+    last = max(i for i, sg in enumerate(segs) if sg[2] == api.SEG_WINDOW)
+    return [(o, n, api.SEG_CURRENT if i == last else kind, sl) for i, (o, n, kind, sl) in enumerate(segs)]
+
+
+@pytest.mark.parametrize("F,h,w,k", [(3, 12, 16, 2), (4, 7, 9, 3), (2, 8, 8, 1)])
+def test_frame_causal_mode_matches_the_oracle(F, h, w, k):
+    """CRC_ATTN_FRAME_CAUSAL on the tensor-core kernel (bf16) and the SIMT kernel (fp32): a
+    query of frame t sees only frames <= t of the current chunk's segment."""
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=40 + F + h, L=1, H=2, F=F, h=h, w=w, k=k)
+    segs = _with_current(segs)
+    Og, lg = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, k, 2.0, 1.0, flags=api.ATTN_FRAME_CAUSAL)
+    Oo, lo = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0, mask_mode="frame")
+    # N(0, 1) queries and keys make single rows peaky: the bf16 kernel is checked against its
+    # rounding model (which takes the same mask), the fp32 kernel against the oracle at 1e-4
+    _check_bf16_against_kernel_model(Og, Oo, Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0, mask_mode="frame")
+    assert np.abs(lg - lo).max() <= 1e-3
+    shp32 = api.shape(1, 2, 128, F, h, w, torch.float32)
+    Os, ls = _run_attn(shp32, Q, Kc, Vc, segs, uv, valid, k, 2.0, 1.0, flags=api.ATTN_FRAME_CAUSAL,
+                       dtype=torch.float32)
+    assert np.abs(Os - Oo).max() <= 1e-4 and np.abs(ls - lo).max() <= 1e-4
+    # the mask changes the earlier frames' rows by far more than the tolerance
+    Oc, _ = _oracle(Q, Kc, Vc, uv, valid, segs, geom, 2.0, 1.0)
+    assert np.abs(Oc - Oo).max() > 5e-2
+
+
+def test_current_segment_without_the_flag_is_a_window_segment_bitwise():
+    shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=44, L=1)
+    a = _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0)
+    b = _run_attn(shp, Q, Kc, Vc, _with_current(segs), uv, valid, geom[3], 2.0, 1.0)
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[1], b[1])
+
+
+def test_frame_causal_mode_at_the_wan13b_shape_sampled():
+    """The Wan-1.3B chunk shape (one layer, 12 heads, 18 720 keys) with the newest window slot
+    as the current chunk: sampled rows of every frame and every head against the oracle."""
+    wl = synth.make_workload(2)
+    _, _, count, slots = _gpu.oracle_retrieve(wl)
+    uv, _, valid, _, _, _ = _gpu.oracle_correspond(wl, slots, count)
+    uv = uv.astype(np.float32)
+    uv[~valid] = 0.0
+    segs = _with_current(wl.segments)
+    g = torch.Generator(device="cuda").manual_seed(45)
+    s = wl.qkv_scale
+    q = (torch.randn(1, wl.Nq, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    kc = (torch.randn(1, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    vc = (torch.randn(1, wl.n_keys, wl.H, wl.d, generator=g, device="cuda") * s).to(torch.bfloat16)
+    shp = api.shape(1, wl.H, wl.d, wl.F, wl.h, wl.w, torch.bfloat16)
+    Og, lg = _run_attn(shp, q, kc, vc, segs, uv, valid, wl.k, wl.lam, wl.sigma, slot_chunk=slots,
+                       flags=api.ATTN_FRAME_CAUSAL)
+    rows = np.random.default_rng(6).choice(wl.Nq, 384, replace=False)
+    rows.sort()
+    assert len(set(rows // (wl.h * wl.w))) == wl.F
+    Qo, Ko, Vo = (t.float().cpu().numpy() for t in (q, kc, vc))
+    Oo, lo = oracle.attention(Qo, Ko, Vo, uv.astype(np.float64), valid, segs, wl.h, wl.w, wl.F, wl.lam, wl.sigma,
+                              slot_chunks=slots, rows=rows, mask_mode="frame")
+    _check_bf16(Og, lg, Oo, lo, rows=rows)
+
+
 # ---------------------------------------------------------------------------- opt-in modes
 def test_gaussian_form_fp32_and_bf16_match_oracle():
     wl = synth.make_workload(1)
@@ -445,7 +508,7 @@ def test_gaussian_form_tensor_core_full_size_sampled_and_against_simt():
 def test_unknown_attention_flags_are_rejected():
     shp, Q, Kc, Vc, segs, uv, valid, geom = _small_case(seed=22, L=1, H=1)
     with pytest.raises(api.CrcError):
-        _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=16)
+        _run_attn(shp, Q, Kc, Vc, segs, uv, valid, geom[3], 2.0, 1.0, flags=32)
 
 
 def _skip_case(seed, far_logit=0.0, invalid_row=None):

@@ -53,6 +53,47 @@ def test_two_rank_timing_reduction(tmp_path):
     assert res[0]["seed"] != res[1]["seed"]
 
 
+def _heads_main(rank, world, port, out_dir):
+    sys.path.insert(0, ROOT)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_21848_gb300 import api
+
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    out = {}
+    for H in (2, 3, 12, 40, 41):
+        h0, nh = api.head_range(H, rank, world)
+        # this rank's view of a [L, N, H, d] tensor is exactly its heads
+        t = torch.arange(2 * 3 * H * 4).reshape(2, 3, H, 4)
+        v = api.head_view(t, h0, nh)
+        assert v.shape[2] == nh and torch.equal(v, t[:, :, h0:h0 + nh])
+        got = [None] * world
+        dist.all_gather_object(got, (h0, nh))
+        out[H] = got
+    dist.barrier()
+    dist.destroy_process_group()
+    with open(os.path.join(out_dir, f"h{rank}.json"), "w") as f:
+        json.dump(out, f)
+
+
+def test_two_ranks_cover_the_heads_disjointly_and_completely(tmp_path):
+    """Each gloo rank takes its head range (api.head_range) and builds its views; the ranges
+    the ranks report to each other tile [0, H) with no overlap and no gap."""
+    world = 2
+    mp.start_processes(_heads_main, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True,
+                       start_method="spawn")
+    res = [json.load(open(tmp_path / f"h{r}.json")) for r in range(world)]
+    assert res[0] == res[1]  # every rank sees the same split
+    for H, ranges in res[0].items():
+        covered = []
+        for h0, nh in ranges:
+            assert nh >= 1
+            covered.extend(range(h0, h0 + nh))
+        assert covered == list(range(int(H))), (H, ranges)  # disjoint, complete, in rank order
+
+
 def test_single_rank_needs_no_process_group():
     sys.path.insert(0, ROOT)
     import bench

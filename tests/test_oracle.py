@@ -648,3 +648,72 @@ def test_gather_repositions_keys_next_to_the_window():
         np.testing.assert_allclose(out[r][0], want, atol=1e-12)
         np.testing.assert_array_equal(out[r][1], pool[j % P, 1])
     assert out[2] is None
+
+
+# ----------------------------------------------------------------------------
+# frame-causal mask inside the current chunk (test mode of the attention)
+# ----------------------------------------------------------------------------
+
+
+def _frame_causal_case(seed=3, F=3, h=2, w=3):
+    g = np.random.default_rng(seed)
+    Nc = F * h * w
+    segs = [(0, Nc, oracle.crc_oracle.SEG_SINK, 0), (Nc, Nc, oracle.crc_oracle.SEG_RETRIEVED, 0),
+            (2 * Nc, Nc, oracle.crc_oracle.SEG_CURRENT, 0)]
+    Nk = 3 * Nc
+    Q = g.standard_normal((1, Nc, 1, 8))
+    K = g.standard_normal((1, Nk, 1, 8))
+    V = g.standard_normal((1, Nk, 1, 8))
+    S = F
+    uv = np.stack([g.uniform(0, w, (Nc, S)), g.uniform(0, h, (Nc, S))], -1)
+    valid = g.uniform(size=(Nc, S)) < 0.7
+    return Q, K, V, uv, valid, segs, (F, h, w)
+
+
+def test_frame_causal_mask_matches_a_double_loop_softmax():
+    Q, K, V, uv, valid, segs, (F, h, w) = _frame_causal_case()
+    lam, sigma = 1.5, 0.8
+    O, lse = oracle.attention(Q, K, V, uv, valid, segs, h, w, F, lam, sigma, mask_mode="frame")
+    Nc, hw = F * h * w, h * w
+    d = Q.shape[-1]
+    for p in range(Nc):
+        tq = p // hw
+        logits, vals = [], []
+        for kk in range(K.shape[1]):
+            seg = kk // Nc
+            loc = kk - seg * Nc
+            if seg == 2 and loc // hw > tq:  # a later frame of the current chunk
+                continue
+            a = sum(Q[0, p, 0, e] * K[0, kk, 0, e] for e in range(d)) / math.sqrt(d)
+            if seg == 1 and valid[p, loc // hw]:
+                x, y = (loc % hw) % w, (loc % hw) // w
+                ux, uy = uv[p, loc // hw]
+                a += lam * -((x - ux) ** 2 + (y - uy) ** 2) / (2 * sigma * sigma)
+            logits.append(a)
+            vals.append(V[0, kk, 0])
+        mx = max(logits)
+        ex = [math.exp(a - mx) for a in logits]
+        tot = sum(ex)
+        ref = sum(e * v for e, v in zip(ex, vals)) / tot
+        np.testing.assert_allclose(O[0, p, 0], ref, rtol=1e-12, atol=1e-12)
+        assert lse[0, 0, p] == pytest.approx(mx + math.log(tot), abs=1e-12)
+
+
+def test_frame_causal_mask_special_cases():
+    # one frame per chunk: nothing to mask, the chunk mode exactly
+    Q, K, V, uv, valid, segs, (F, h, w) = _frame_causal_case(seed=4, F=1, h=3, w=3)
+    a = oracle.attention(Q, K, V, uv, valid, segs, h, w, F, 2.0, 1.0, mask_mode="frame")
+    b = oracle.attention(Q, K, V, uv, valid, segs, h, w, F, 2.0, 1.0)
+    np.testing.assert_array_equal(a[0], b[0])
+    # only the current chunk: frame-0 queries attend to the frame-0 keys alone, the last frame's
+    # queries to every key (the chunk mode)
+    Q, K, V, uv, valid, _, (F, h, w) = _frame_causal_case(seed=5)
+    Nc, hw = F * h * w, h * w
+    cur = [(0, Nc, oracle.crc_oracle.SEG_CURRENT, 0)]
+    O = oracle.attention(Q, K[:, :Nc], V[:, :Nc], uv, valid, cur, h, w, F, 2.0, 1.0, mask_mode="frame")[0]
+    first = oracle.attention(Q[:, :hw], K[:, :hw], V[:, :hw], uv, valid, [(0, hw, oracle.crc_oracle.SEG_WINDOW, 0)],
+                             h, w, F, 2.0, 1.0)[0]
+    np.testing.assert_allclose(O[:, :hw], first, rtol=1e-13, atol=1e-13)
+    full = oracle.attention(Q, K[:, :Nc], V[:, :Nc], uv, valid, cur, h, w, F, 2.0, 1.0)[0]
+    np.testing.assert_array_equal(O[:, (F - 1) * hw:], full[:, (F - 1) * hw:])
+    assert np.abs(O - full).max() > 1e-3  # the mask does change the earlier frames
