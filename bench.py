@@ -213,9 +213,9 @@ def run_step(W, stream, ev=None):
 LAUNCHES_PER_STEP = 5
 
 # DRAM bytes (read + write) per layer of attn_tc_kernel at the Wan-1.3B chunk shape, from one
-# ncu capture of a 2-layer launch (283.8 MB / 2); traffic grows in proportion to layers.
-# Valid only for that shape and the kernel version it was captured on.
-ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.9e6}
+# ncu capture of a 2-layer launch of the current kernel (259.6 + 23.9 MB / 2); traffic grows in
+# proportion to layers.  Valid only for that shape and the kernel version it was captured on.
+ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.77e6}
 
 
 # ---------------------------------------------------------------------------- ranks
@@ -275,13 +275,21 @@ def run_e2e(W, stream, steps: int):
     h2d_s.wait_stream(stream)
     d2h_s.wait_stream(stream)
 
+    # per-step timeline: uploads and downloads on the copy stream, the step on the compute stream
+    T = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    up = [(T(), T()) for _ in range(steps)]
+    dn = [(T(), T()) for _ in range(steps)]
+    cp = [(T(), T()) for _ in range(steps)]
+
     def upload(i):
         b = i % NB
         with torch.cuda.stream(h2d_s):
             if i >= NB:
                 h2d_s.wait_event(done[b])  # step i-NB has finished reading buffer b
+            up[i][0].record(h2d_s)
             for k in E2E_INPUTS:
                 dev[b][k].copy_(host_in[k], non_blocking=True)
+            up[i][1].record(h2d_s)
             in_ready[b].record(h2d_s)
 
     for i in range(min(NB - 1, steps)):
@@ -293,11 +301,15 @@ def run_e2e(W, stream, steps: int):
         stream.wait_event(in_ready[b])
         if i >= NB:
             stream.wait_event(out_read[b])  # O of step i-NB has left buffer b
+        cp[i][0].record(stream)
         run_step(dev[b], stream)
+        cp[i][1].record(stream)
         done[b].record(stream)
         with torch.cuda.stream(d2h_s):
             d2h_s.wait_event(done[b])
+            dn[i][0].record(d2h_s)
             host_out[b].copy_(dev[b]["o"], non_blocking=True)
+            dn[i][1].record(d2h_s)
             out_read[b].record(d2h_s)
     stream.wait_stream(h2d_s)
     stream.wait_stream(d2h_s)
@@ -305,7 +317,26 @@ def run_e2e(W, stream, steps: int):
     torch.cuda.synchronize()
     h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + W["frames"].nbytes
     d2h = host_out[0].numel() * host_out[0].element_size()
-    return e0.elapsed_time(e1) / 1e3 / steps, h2d, d2h
+    med = lambda xs: statistics.median(xs) if xs else None  # noqa: E731
+    timeline = {
+        "compute_ms": med([a.elapsed_time(b) for a, b in cp]),
+        "upload_ms": med([a.elapsed_time(b) for a, b in up]),
+        "download_ms": med([a.elapsed_time(b) for a, b in dn]),
+        # compute stream idle between the end of step i-1 and the start of step i (waiting for inputs
+        # or a free buffer set)
+        "compute_gap_ms": med([cp[i - 1][1].elapsed_time(cp[i][0]) for i in range(1, steps)]),
+        "compute_gap_max_ms": max([cp[i - 1][1].elapsed_time(cp[i][0]) for i in range(1, steps)], default=None),
+        "compute_gap_total_ms": sum(cp[i - 1][1].elapsed_time(cp[i][0]) for i in range(1, steps)),
+        # the longest waits with the duration of the upload the waiting step needed
+        "longest_gaps": sorted(({"step": i, "gap_ms": cp[i - 1][1].elapsed_time(cp[i][0]),
+                                 "its_upload_ms": up[i][0].elapsed_time(up[i][1]),
+                                 "upload_start_to_compute_start_ms": up[i][0].elapsed_time(cp[i][0])}
+                                for i in range(1, steps)), key=lambda r: -r["gap_ms"])[:4],
+        "upload_ms_max": max(a.elapsed_time(b) for a, b in up),
+        "download_ms_max": max(a.elapsed_time(b) for a, b in dn),
+        "note": "medians per step from CUDA events on the copy stream (uploads, downloads) and the compute stream",
+    }
+    return e0.elapsed_time(e1) / 1e3 / steps, h2d, d2h, timeline
 
 
 def link_gbs(W, reps: int = 3):
@@ -767,15 +798,16 @@ def main():
 
     barrier()
     with ClockSampler(local) as clk_e2e:
-        e2e_s, h2d, d2h = run_e2e(W, stream, max(3, args.steps))  # as many steps as the device timing
+        e2e_s, h2d, d2h, e2e_timeline = run_e2e(W, stream, max(3, args.steps))  # as many steps as the device timing
     link = link_gbs(W)
     e2e_s = max_over_ranks(e2e_s, world, device)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
-    sweep = shapes = modes = stream_ctx = None
+    sweep = shapes = modes = stream_ctx = gsweep = None
     if not args.no_context:
-        from sweeps import correspond_sweep
+        from sweeps import correspond_sweep, gather_sweep
 
+        gsweep = gather_sweep(device)
         sweep = correspond_sweep(device)
         sweep["iid_depth"] = {key: val for key, val in correspond_sweep(device, depth="iid").items()
                               if key in ("ms", "gbs", "eager_ms", "valid_fraction")}
@@ -797,7 +829,14 @@ def main():
     if sweep is not None:
         hbm_rooflines["correspond_sweep"] = {"kernel": "correspond_kernel", "gbs": sweep["gbs"], "bytes": sweep["bytes"],
                                              "what": "126 MB reprojection sweep (4 x 180 x 320 queries, 32 frames)"}
-    for key in ("retrieve_gather", "cache_update", "correspond_sweep"):
+    if gsweep is not None:
+        hbm_rooflines["rope_gather"] = {"kernel": "gather_kernel (re-positioned keys)", "gbs": gsweep["rope"]["gbs"],
+                                        "bytes": gsweep["rope"]["bytes"],
+                                        "what": "crc_gather of one chunk, 30 layers, 22 interleaved temporal pairs "
+                                                "rotated in every key row"}
+        hbm_rooflines["plain_gather"] = {"kernel": "gather_kernel", "gbs": gsweep["plain"]["gbs"],
+                                         "bytes": gsweep["plain"]["bytes"], "what": "the same gather unrotated"}
+    for key in ("retrieve_gather", "cache_update", "correspond_sweep", "rope_gather", "plain_gather"):
         if key in hbm_rooflines:
             hbm_rooflines[key]["frac"] = hbm_rooflines[key]["gbs"] / peaks["hbm"]
     line = {
@@ -837,6 +876,7 @@ def main():
                 "pipelining": f"{E2E_BUFFERS} device buffer sets; on one copy stream, uploads run up to "
                               f"{E2E_BUFFERS - 1} steps ahead and downloads trail, overlapping the kernels",
                 "link_gbs": link,
+                "timeline": e2e_timeline,
                 "clocks": clk_e2e.summary(),
                 "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6},
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
@@ -846,7 +886,8 @@ def main():
     }
     if context is not None:
         line["context"] = {"sdpa": context, "note": "PyTorch SDPA on the same Q/K/V, not part of the path",
-                           "correspond_sweep": sweep, "other_shapes": shapes, "opt_in_modes": modes,
+                           "correspond_sweep": sweep, "gather_sweep": gsweep, "other_shapes": shapes,
+                           "opt_in_modes": modes,
                            "stream": stream_ctx}
         if sweep is not None:
             sweep["frac_of_hbm_peak"] = sweep["gbs"] / peaks["hbm"]

@@ -17,8 +17,8 @@
 // The launch allows programmatic stream serialization: a block first does the work
 // that depends on its arguments alone, then waits for the grid before it
 // (griddepcontrol.wait) before it reads bank data or depths or writes an output, and
-// once its prologue is done it lets the next grid begin its launch, so that launch
-// latency overlaps the running grid.
+// it lets the next grid begin its launch as soon as it starts, so that launch latency
+// overlaps the running grid.  Depths are read through the read-only data path.
 #include <math.h>
 
 #include "internal.cuh"
@@ -106,6 +106,9 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   __shared__ int src_off[kMaxS];
   __shared__ float tgt_RK[CRC_MAX_FRAMES][9];  // R_t K_t^-1
   __shared__ double tgt_c[CRC_MAX_FRAMES][3];  // c_t
+  // the next grid may begin its launch at once: this grid is one wave, so nothing of it
+  // waits for SM space, and the next grid's blocks wait for this one before they read
+  asm volatile("griddepcontrol.launch_dependents;");
   const int S = a.k * a.F;
   const int hw = a.h * a.w;
   const int Nq = a.F * hw;
@@ -218,7 +221,6 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   }
   __syncthreads();
 
-  asm volatile("griddepcontrol.launch_dependents;");  // the next grid may begin its launch
   if (q >= q_end) return;
   int t = q / hw;
   int iy = (q - t * hw) / a.w;
@@ -241,7 +243,7 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
   Idx o = (Idx)q * (Idx)S + (Idx)s0;
   const Idx o_step = (Idx)R * (Idx)S;
   for (; q < q_end; q += R, o += o_step) {
-    const float zn = q + R < q_end ? a.depth[q + R] : 0.f;  // next query's depth, in flight meanwhile
+    const float zn = q + R < q_end ? __ldg(a.depth + q + R) : 0.f;  // next query's depth, in flight meanwhile
     const float u0 = (float)jx;
     const bool z_ok = (z > 0.f) & (z < INFINITY);
     float ux[P], uy[P], X2[P];
@@ -279,7 +281,7 @@ __global__ void __launch_bounds__(256, 4) correspond_kernel(const __grid_constan
     if (VIS) {
       float ds[P];
 #pragma unroll
-      for (int p = 0; p < P; ++p) ds[p] = *(ok[p] ? a.bank_depth + (doff[p] + cell[p]) : a.depth + q);
+      for (int p = 0; p < P; ++p) ds[p] = __ldg(ok[p] ? a.bank_depth + (doff[p] + cell[p]) : a.depth + q);
 #pragma unroll
       for (int p = 0; p < P; ++p) {
         ok[p] = ok[p] & (X2[p] <= one_eps * ds[p]);

@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(kTopkThreads) retrieve_topk_kernel(const __gri
 // a programmatic dependent launch, and griddepcontrol.wait holds it until the top-k
 // results are visible; launched on its own, the wait returns at once.
 template <bool ROPE>
-__global__ void __launch_bounds__(256, ROPE ? 2 : 4) gather_kernel(const __grid_constant__ GatherOnlyArgs a) {
+__global__ void __launch_bounds__(256, 4) gather_kernel(const __grid_constant__ GatherOnlyArgs a) {
   __shared__ GatherPlan plan;
   asm volatile("griddepcontrol.wait;" ::: "memory");
   if (threadIdx.x < a.k) plan.chunk[threadIdx.x] = a.d_idx[threadIdx.x];
