@@ -460,22 +460,35 @@ def sdpa_context(W, flops: float, iters: int = 5):
 
 # ---------------------------------------------------------------------------- oracle arm
 def other_shapes(device, seed: int, iters: int = 5):
-    """The attention call alone on the other bf16 shapes: Wan-1.3B with k = 3 (28 080 keys, 30
-    layers batched) and the 14B-class 720p shape (40 heads, 10 800 queries, 64 800 keys, one
-    layer).  One full step first fills each cache and its correspondences through the path;
-    then the attention is timed with CUDA events.  Context for how the kernel holds beyond the
-    headline shape."""
+    """The other workloads: Wan-1.3B with k = 3 (28 080 keys, 30 layers batched, a bank of 2000
+    chunks), the 14B-class 720p shape (40 heads, 10 800 queries, 64 800 keys, one layer, a bank
+    of 500) and the tiny fp32 case.  Whole chunk steps are timed first with CUDA events around
+    each stage (update, retrieval with its scoring and gather, reprojection, attention); then the
+    attention call alone.  Context for how the path holds beyond the headline shape."""
     import torch
 
     from paper_2607_21848_gb300 import api
 
     out = {}
-    for cfg, layers in ((3, 30), (4, 1)):  # synth workloads: Wan-1.3B k = 3, and 14B-class 720p
+    for cfg, layers in ((3, 30), (4, 1), (1, 1)):  # synth workloads: Wan-1.3B k = 3, 14B-class 720p, tiny fp32
         W = setup(cfg, layers, device, seed)
         wl = W["wl"]
         stream = torch.cuda.current_stream()
         run_step(W, stream)
         flops = algorithmic(W)["flops"]
+        alg = algorithmic(W)
+        for _ in range(2):
+            run_step(W, stream)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(iters)]
+        for i in range(iters):
+            run_step(W, stream, evs[i])
+        torch.cuda.synchronize()
+        st = {nm: statistics.median(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(iters))
+              for j, nm in enumerate(("update", "retrieve", "correspond", "attention"))}
+        step = {"stage_ms": st, "retrieve_gbs": alg["gather_bytes"] / st["retrieve"] / 1e6,
+                "update_gbs": alg["update_bytes"] / st["update"] / 1e6,
+                "correspond_gbs": alg["reproj_bytes"] / st["correspond"] / 1e6,
+                "bank": wl.bank_size, "gather_bytes": alg["gather_bytes"]}
 
         def attn():
             api.crc_biased_attention(W["shape"], W["q"], W["cache"], W["o"], None, W["uv"], W["valid"], wl.k,
@@ -494,7 +507,7 @@ def other_shapes(device, seed: int, iters: int = 5):
         if int(W["status"].item()) != 0:
             raise RuntimeError(f"attention status {int(W['status'].item())} on config {cfg}")
         out[wl.name] = {"layers": layers, "heads": wl.H, "queries": wl.Nq, "keys": wl.n_keys, "k": wl.k,
-                               "ms": ms, "tflops": flops / ms / 1e9}
+                        "dtype": wl.dtype, "ms": ms, "tflops": flops / ms / 1e9, "step": step}
         del W
         torch.cuda.empty_cache()
     return out
@@ -692,6 +705,79 @@ def oracle_sample(cfg_id: int, layers: int, budget_s: float):
                 step_s=step_s, heads=heads, threads=os.cpu_count())
 
 
+def oracle_stages(cfg_id: int, budget_s: float = 4.0):
+    """The fp64 oracle's stages for one chunk step of a workload, timed separately (run in a
+    child process whose BLAS and OpenMP pools have one thread): the pose summaries and Eq. 1
+    retrieval over the bank, the gather of the retrieved chunks' K/V (all layers), the
+    reprojection of every query into every retrieved frame, and the attention, whose time is
+    extrapolated from whole (layer, head) rows sampled for `budget_s`."""
+    import oracle
+    import synth
+
+    wl = synth.make_workload(cfg_id, layers=30 if cfg_id == 2 else None)  # config 2: the 30-layer chunk step
+    out = {"workload": wl.name, "layers": wl.L}
+    t0 = time.perf_counter()
+    bc = np.zeros((wl.bank_size, 3))
+    bv = np.zeros((wl.bank_size, 3))
+    for j in range(wl.bank_size):
+        bc[j], bv[j] = oracle.chunk_pose(wl.bank_frames.R[j], wl.bank_frames.c[j])
+    cn, vn = oracle.chunk_pose(wl.cur_frames.R, wl.cur_frames.c)
+    idx, _, count = oracle.retrieve(bc, bv, cn, vn, wl.n, wl.E, wl.w_v, wl.tau_c, wl.cos_tau_v, wl.delta, wl.k)
+    slots = oracle.fill_slots(idx, count, -1, 0)
+    out["retrieve_s"] = time.perf_counter() - t0
+    g = np.random.default_rng(0)
+    row = wl.H * wl.d
+    slab = g.standard_normal((1, 2, wl.L, wl.Nc, wl.H, wl.d)).astype(np.float32)
+    t0 = time.perf_counter()
+    for r in range(wl.k):
+        oracle.gather(slab, np.array([0]), 1)
+    out["gather_s"] = time.perf_counter() - t0
+    out["gather_bytes"] = 2 * 2 * wl.k * wl.L * wl.Nc * row * (2 if wl.dtype == "bf16" else 4)
+    S = wl.k * wl.F
+    Ks, Rs, cs = np.zeros((S, 3, 3)), np.zeros((S, 3, 3)), np.zeros((S, 3))
+    ds = np.ones((S, wl.h, wl.w), dtype=np.float32)
+    ok = np.zeros(S, bool)
+    for r, j in enumerate(slots):
+        for f in range(wl.F):
+            fr = wl.bank_frames[max(j, 0)]
+            Ks[r * wl.F + f], Rs[r * wl.F + f], cs[r * wl.F + f] = fr.K[f], fr.R[f], fr.c[f]
+            if j >= 0:
+                ds[r * wl.F + f] = wl.depth_of(j)[f]
+                ok[r * wl.F + f] = True
+    cur = wl.cur_frames
+    dep = wl.depth_of(wl.n)
+    t0 = time.perf_counter()
+    uv, _, valid = oracle.correspond(dep, cur.K, cur.R, cur.c, ds, Ks, Rs, cs, wl.eps, source_ok=ok)
+    out["correspond_s"] = time.perf_counter() - t0
+    Q = g.standard_normal((1, wl.Nq, 1, wl.d)) * wl.qkv_scale
+    Kc = g.standard_normal((1, wl.n_keys, 1, wl.d)) * wl.qkv_scale
+    Vc = g.standard_normal((1, wl.n_keys, 1, wl.d)) * wl.qkv_scale
+    rows_done, t_attn, blk = 0, 0.0, 64
+    while t_attn < budget_s and rows_done < wl.Nq:
+        rows = np.arange(rows_done, min(rows_done + blk, wl.Nq))
+        t0 = time.perf_counter()
+        oracle.attention(Q, Kc, Vc, uv, valid, wl.segments, wl.h, wl.w, wl.F, wl.lam, wl.sigma, slot_chunks=slots,
+                         rows=rows)
+        t_attn += time.perf_counter() - t0
+        rows_done += rows.shape[0]
+    out["attention_s"] = t_attn / rows_done * wl.Nq * wl.H * wl.L
+    out["attention_rows_sampled"] = rows_done
+    out["step_s"] = out["retrieve_s"] + out["gather_s"] + out["correspond_s"] + out["attention_s"]
+    return out
+
+
+def one_thread_oracle_stages(configs=(1, 2)):
+    """oracle_stages of each workload in a child process with single-threaded BLAS and OpenMP."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    out = {}
+    for cfg in configs:
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-stages", str(cfg)], env=env,
+                           capture_output=True, text=True, timeout=600)
+        lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+        out[str(cfg)] = json.loads(lines[-1]) if r.returncode == 0 and lines else {"error": r.stderr[-300:]}
+    return out
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -740,11 +826,15 @@ def main():
     ap.add_argument("--layers", type=int, default=30)
     ap.add_argument("--impl", default="crc", choices=["crc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-stages", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--no-context", action="store_true",
                     help="skip the context block: PyTorch SDPA comparators, the reprojection sweep, the opt-in "
                          "attention modes, the loop-closure stream and the other shapes")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.oracle_stages:
+        print(json.dumps(oracle_stages(args.oracle_stages)))
+        return
     if args.impl == "reference":
         run_reference(args)
         return
@@ -902,6 +992,7 @@ def main():
                       f"{cb['rows']} attention rows from {cb['heads']} (layer, head) problems of {wl.Nq} rows, "
                       f"each against all {wl.n_keys} keys ({cb['t_attn']:.1f} s); TFLOP/s = sampled attention "
                       f"FLOP / sampled time; a full step extrapolates to {cb['step_s']:.0f} s"}
+        line["cpu_baseline"]["one_thread_stages"] = one_thread_oracle_stages()
     if rank == 0:
         print(json.dumps(line))
     if world > 1:
