@@ -389,12 +389,13 @@ crc_status crc_correspond(const crc_shape* shape, const crc_frame* cur, const fl
  * accumulation, in either bias form; fp32 or CRC_ATTN_SIMT run the SIMT kernel in fp32.
  * Eq. 2 on the tensor-core kernel: the bias is added to S by the tensor core itself, as
  * a K = 16 extension of q.k (a rank-4 expansion of ||u_k - u^||^2 about the frame centre).
- * Its terms cancel near the correspondence, so its error grows with the grid: at most
- * crc_bias_expansion_bound(lambda, sigma, h, w) = 2^-23 C (w^2 + h^2) in base-2 logit
- * units, C = lambda log2(e) / (2 sigma^2).  Where that exceeds 2^-9 (the bf16 rounding
- * of the softmax weights; e.g. lambda / sigma^2 > 2.69 on a 45 x 80 grid, > 6.3 on
- * 30 x 52) the kernel adds the bias per score in the softmax instead, exact to fp32
- * rounding, at a lower throughput; CRC_ATTN_BIAS_DIRECT selects that everywhere.
+ * Its strength is taken to 16 significant bits (lambda scaled by 1 + delta, |delta| <=
+ * 2^-17), and its terms cancel near the correspondence, so its error grows with the
+ * grid: at most crc_bias_expansion_bound(lambda, sigma, h, w) = 2^-24 C (w^2 + h^2) in
+ * base-2 logit units, C = lambda log2(e) / (2 sigma^2).  Where that exceeds 2^-9 (the
+ * bf16 rounding of the softmax weights; e.g. lambda / sigma^2 > 5.39 on a 45 x 80 grid,
+ * > 12.6 on 30 x 52) the kernel adds the bias per score in the softmax instead, exact to
+ * fp32 rounding, at a lower throughput; CRC_ATTN_BIAS_DIRECT selects that everywhere.
  * The tensor-core kernel takes at most 640 KV tiles of 128 keys per call (each
  * segment is cut into tiles from its start, a retrieved segment per frame: up to
  * 81 920 keys) and h*w <= 65535; beyond that the call returns CRC_ERR_UNSUPPORTED
@@ -481,7 +482,8 @@ typedef struct {
 crc_status crc_chunk_step(const crc_step_plan* plan, const crc_step* d_step, cudaStream_t s);
 
 /* Bound on the error of the tensor-core expansion of the Eq. 2 bias on an h x w grid,
- * in base-2 logit units: 2^-23 lambda log2(e) / (2 sigma^2) (w^2 + h^2); +inf where
+ * in base-2 logit units: 2^-24 lambda log2(e) / (2 sigma^2) (w^2 + h^2), besides the
+ * consistent 2^-17 scale of the bias strength; +inf where
  * the key coordinates are not exact in bf16 (w or h above 256, or
  * (w-1)^2 + (h-1)^2 >= 2^16), which always takes the per-score form.  Host only. */
 double crc_bias_expansion_bound(float lambda, float sigma, int32_t h, int32_t w);

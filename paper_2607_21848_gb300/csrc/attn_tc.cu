@@ -12,12 +12,13 @@
 // (x' = x - (w-1)/2, y' = y - (h-1)/2) and A = lambda log2(e) / (2 sigma^2) in base-2
 // units (0 when the pair is invalid), the bias of Eq. 2 expands as
 //   A (q_k - 2 ux' x'_k - 2 uy' y'_k + ux'^2 + uy'^2),   q_k = x'_k^2 + y'_k^2,
-// a dot product of a 4-vector per query row with a 4-vector per key.  Each query
-// coefficient is split into three bf16 terms (hi + mid + lo, ~24 bits) and q_k into
-// two (exact: x', y' are half-integers), giving a K = 16 extension of the QK^T
-// contraction whose products are exact in fp32:
-//   query row: [a0h a0h a0m a0m a0l a0l a1h a1m a1l a2h a2m a2l a3h a3m a3l 1]
-//   key row:   [qh  ql  qh  ql  qh  ql  x'  x'  x'  y'  y'  y'  1   1   1   M]
+// a dot product of a 4-vector per query row with a 4-vector per key.  A is rounded to
+// two bf16 terms (A'), the other query coefficients are formed from A' in double-fp32
+// arithmetic and split into four (linear terms) or three (constant term) bf16 terms,
+// and q_k into two (exact: x', y' are half-integers), giving a K = 16 extension of the
+// QK^T contraction whose products are exact:
+//   query row: [ah ah al al | c1 c1 c1 c1 | c2 c2 c2 c2 | c3 c3 c3 | 1]
+//   key row:   [qh ql qh ql | x' x' x' x' | y' y' y' y' | 1  1  1  | M]
 // The last column masks keys past the tile's end (M = -2^100, else 0); an unbiased
 // tile has zeros in the first fifteen key columns.  One extra tcgen05.mma
 // (M = N = 128, K = 16, no-swizzle K-major operands) per query tile adds it to S,
@@ -56,16 +57,16 @@
 //
 // Accuracy of the expansion.  Its large terms (A q_k, 2 A ux' x'_k, ...) cancel to
 // A d^2 near the correspondence, so its absolute error grows with the grid: in base-2
-// logit units it stays below 2^-23 C (w^2 + h^2), C = lambda log2(e) / (2 sigma^2).
-// The error comes from rounding the query coefficients -2A ux', -2A uy' and
-// A (ux'^2 + uy'^2) to fp32 before their (exact) three-term split: a CPU model of
-// those steps alone gives 0.43-0.67 x 2^-24 C (w^2 + h^2), and this GPU measures
-// 0.49-0.64 of that unit, so the tensor core's fp32 sum adds little.  The key terms
-// are exact for grids up to 256 a side with (w-1)^2 + (h-1)^2 < 2^16.  Where the
-// bound exceeds 2^-9 -- the bf16 rounding of P -- or the grid is larger, the host
-// selects the direct form (MODE = DIRECT): the K = 16 operand carries only the mask
-// and the softmax adds C d^2 to every biased score from the key's cell, exact to
-// fp32 rounding, at a lower throughput.
+// logit units it stays below 2^-24 C (w^2 + h^2), C = lambda log2(e) / (2 sigma^2), on
+// top of the consistent 2^-17 scale of A'.  With the coefficients formed in double-fp32
+// their representation contributes 0.6-2.4 x 2^-28 C (w^2 + h^2) (a CPU model of these
+// steps); this GPU measures 3.8-6.6 x 2^-28 C (w^2 + h^2) in all, the rest being the
+// tensor core's own fp32 sum of the 16 products.  (Coefficients rounded to fp32 before
+// the split measured 8-10 x 2^-28.)  The key terms are exact for grids up to 256 a
+// side with (w-1)^2 + (h-1)^2 < 2^16.  Where the bound exceeds 2^-9 -- the bf16
+// rounding of P -- or the grid is larger, the host selects the direct form (MODE =
+// DIRECT): the K = 16 operand carries only the mask and the softmax adds C d^2 to
+// every biased score from the key's cell, exact to fp32 rounding, at a lower throughput.
 //
 // The opt-in additive-Gaussian form (lambda exp(-d^2 / (2 sigma^2)) on the same
 // columns) has no low-rank expansion either: its instantiation (MODE = GAUSS) adds
@@ -194,15 +195,30 @@ __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.a
 __device__ __forceinline__ uint32_t bf16_bits(float v) {
   return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v));
 }
-// v ~= hi + mid + lo in bf16 (each term rounded to nearest from the remainder)
-__device__ __forceinline__ void split3(float v, uint32_t& h, uint32_t& m, uint32_t& l) {
-  const __nv_bfloat16 bh = __float2bfloat16_rn(v);
-  const float r1 = v - __bfloat162float(bh);
-  const __nv_bfloat16 bm = __float2bfloat16_rn(r1);
-  const float r2 = r1 - __bfloat162float(bm);
-  h = (uint32_t)__bfloat16_as_ushort(bh);
-  m = (uint32_t)__bfloat16_as_ushort(bm);
-  l = bf16_bits(r2);
+// Error-free transformations in fp32: each operation rounded once, nothing contracted.
+__device__ __forceinline__ void two_prod(float a, float b, float& p, float& e) {  // a b = p + e exactly
+  p = __fmul_rn(a, b);
+  e = __fmaf_rn(a, b, -p);
+}
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {  // a + b = s + e exactly
+  s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+// hi + lo (|lo| well below |hi|) as N bf16 terms, each the nearest bf16 to what remains;
+// lo joins the remainder after the first term.  The remainder after term i is exact in
+// fp32, so the error is the one rounding that folds lo in (2^-32 of hi) plus what the
+// last term leaves (2^-26 of hi for N = 3, 2^-35 for N = 4).
+template <int N>
+__device__ __forceinline__ void split_df(float hi, float lo, uint32_t (&t)[N]) {
+  float r = hi;
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
+    const __nv_bfloat16 b = __float2bfloat16_rn(r);
+    t[i] = (uint32_t)__bfloat16_as_ushort(b);
+    r = __fsub_rn(r, __bfloat162float(b));
+    if (i == 0) r = __fadd_rn(r, lo);
+  }
 }
 // Write one 16-element bf16 row (given as 8 packed words) of a no-swizzle K-major
 // 128 x 16 operand: 8-row x 16-byte core matrices, K halves 128 bytes apart,
@@ -235,23 +251,44 @@ __device__ __forceinline__ Corr load_corr(const AttnArgs& a, const TileInfo* til
   return c;
 }
 
-// Query-side bias operand row for source frame A of `c` (raw score units).
+// Query-side bias operand row for source frame A of `c` (raw score units).  The bias
+// strength is taken as A' = two bf16 terms of A (16 bits; A' = A (1 + delta), |delta| <=
+// 2^-17, a consistent scale of the whole bias) and every coefficient is formed from A' in
+// double-fp32 arithmetic before its split: -2 A' ux' and -2 A' uy' into four bf16 terms,
+// A' (ux'^2 + uy'^2) into three.
+//   query row: [ah ah al al | c1 c1 c1 c1 | c2 c2 c2 c2 | c3 c3 c3 | 1]
+//   key row:   [qh ql qh ql | x' x' x' x' | y' y' y' y' | 1  1  1  | M]
 __device__ __forceinline__ void aug_query_row(const Corr& c, float xc, float yc, float inv_sc, uint32_t (&w)[8]) {
-  const float A = c.cA * inv_sc;
-  const float ux = c.uxA - xc, uy = c.uyA - yc;
-  uint32_t a0[3], a1[3], a2[3], a3[3];
-  split3(A, a0[0], a0[1], a0[2]);
-  split3(-2.f * A * ux, a1[0], a1[1], a1[2]);
-  split3(-2.f * A * uy, a2[0], a2[1], a2[2]);
-  split3(A * fmaf(ux, ux, uy * uy), a3[0], a3[1], a3[2]);
-  w[0] = a0[0] | (a0[0] << 16);
-  w[1] = a0[1] | (a0[1] << 16);
-  w[2] = a0[2] | (a0[2] << 16);
-  w[3] = a1[0] | (a1[1] << 16);
-  w[4] = a1[2] | (a2[0] << 16);
-  w[5] = a2[1] | (a2[2] << 16);
-  w[6] = a3[0] | (a3[1] << 16);
-  w[7] = a3[2] | (bf16_bits(1.f) << 16);  // mask column
+  const float A = __fmul_rn(c.cA, inv_sc);
+  const __nv_bfloat16 ah = __float2bfloat16_rn(A);
+  const float ahf = __bfloat162float(ah);
+  const __nv_bfloat16 al = __float2bfloat16_rn(__fsub_rn(A, ahf));
+  const float alf = __bfloat162float(al);
+  const float ux = __fsub_rn(c.uxA, xc), uy = __fsub_rn(c.uyA, yc);
+  float p, e;
+  uint32_t t1[4], t2[4], t3[3];
+  // -2 A' u = -2 (ah u + al u): the first product exactly, the second (2^-9 of it) rounded once
+  two_prod(ahf, ux, p, e);
+  split_df<4>(-2.f * p, -2.f * __fmaf_rn(alf, ux, e), t1);
+  two_prod(ahf, uy, p, e);
+  split_df<4>(-2.f * p, -2.f * __fmaf_rn(alf, uy, e), t2);
+  // A' (ux^2 + uy^2), the sum of squares carried as two fp32 terms
+  float sx, ex, sy, ey, sq, es;
+  two_prod(ux, ux, sx, ex);
+  two_prod(uy, uy, sy, ey);
+  two_sum(sx, sy, sq, es);
+  const float sl = __fadd_rn(__fadd_rn(ex, ey), es);
+  two_prod(ahf, sq, p, e);
+  split_df<3>(p, __fmaf_rn(ahf, sl, __fmaf_rn(alf, sq, e)), t3);
+  const uint32_t hb = (uint32_t)__bfloat16_as_ushort(ah), lb = (uint32_t)__bfloat16_as_ushort(al);
+  w[0] = hb | (hb << 16);
+  w[1] = lb | (lb << 16);
+  w[2] = t1[0] | (t1[1] << 16);
+  w[3] = t1[2] | (t1[3] << 16);
+  w[4] = t2[0] | (t2[1] << 16);
+  w[5] = t2[2] | (t2[3] << 16);
+  w[6] = t3[0] | (t3[1] << 16);
+  w[7] = t3[2] | (bf16_bits(1.f) << 16);  // mask column
 }
 
 // fp32 <-> int keys with the same order, for shared-memory atomic min / max
@@ -489,12 +526,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t qh = bf16_bits(q);
           const uint32_t ql = bf16_bits(q - __bfloat162float(__ushort_as_bfloat16((unsigned short)qh)));
           const uint32_t xb = bf16_bits(xr), yb = bf16_bits(yr);
-          w[0] = qh | (ql << 16);
+          w[0] = qh | (ql << 16);  // [qh ql qh ql | x' x4 | y' x4 | 1 1 1 | M]
           w[1] = w[0];
-          w[2] = w[0];
-          w[3] = xb | (xb << 16);
-          w[4] = xb | (yb << 16);
-          w[5] = yb | (yb << 16);
+          w[2] = xb | (xb << 16);
+          w[3] = w[2];
+          w[4] = yb | (yb << 16);
+          w[5] = w[4];
           w[6] = one | (one << 16);
           w[7] = one | (mask << 16);
         }
@@ -859,7 +896,7 @@ double bias_expansion_bound(float lambda, float sigma, int h, int w) {
   // terms) exactly in bf16 only while 2|x'|, 2|y'| < 256 and 4q < 2^16
   if (w > 256 || h > 256 || (int64_t)(w - 1) * (w - 1) + (int64_t)(h - 1) * (h - 1) >= 65536) return INFINITY;
   const double C = (double)lambda * 1.4426950408889634 / (2.0 * (double)sigma * (double)sigma);
-  return C * ((double)w * w + (double)h * h) * 0x1p-23;
+  return C * ((double)w * w + (double)h * h) * 0x1p-24;
 }
 
 // The kernel's limits: bf16, d = 128, at most kMaxTiles KV tiles (each segment cut

@@ -5,10 +5,11 @@ rounding steps the kernel takes, in numpy float32 / bfloat16 emulation, so that 
 tests can tell which part of the kernel's deviation from the oracle each step
 explains.  It shares no code with the CUDA library.
 
-  expansion_terms    the K = 16 bias extension of q.k: the query-side coefficients
-                     A, -2A ux', -2A uy', A(ux'^2 + uy'^2) rounded in fp32 and split
-                     into three bf16 terms each, the key-side q_k (two bf16 terms),
-                     x', y'; their products summed exactly (fp64).
+  expansion_terms    the K = 16 bias extension of q.k: A rounded to two bf16 terms (A'),
+                     the query-side coefficients -2A' ux', -2A' uy', A'(ux'^2 + uy'^2)
+                     formed in double-fp32 and split into 4, 4 and 3 bf16 terms, the
+                     key-side q_k (two bf16 terms), x', y'; their products summed
+                     exactly (fp64).
   attention_model    the softmax protocol per 128-key tile (tile cut per segment and,
                      in retrieved segments, per frame; the stale row max refreshed
                      only when it grows by more than 2^8; P = 2^(s sc - m) rounded to
@@ -28,12 +29,13 @@ f32 = np.float32
 
 
 def bf16(x):
-    """Round float32 values to bfloat16 (nearest even), returned as float32."""
-    a = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+    """Round float32 values to bfloat16 (nearest even), returned as float32 of x's shape."""
+    x = np.asarray(x, dtype=np.float32)
+    a = np.ascontiguousarray(x).reshape(-1)
     u = a.view(np.uint32).astype(np.uint64)
     r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
     out = r.astype(np.uint32).view(np.float32)
-    return np.where(np.isfinite(a), out, a)
+    return np.where(np.isfinite(a), out, a).reshape(x.shape)
 
 
 def split3(v):
@@ -47,6 +49,34 @@ def split3(v):
     return hi.astype(np.float64) + mid.astype(np.float64) + lo.astype(np.float64)
 
 
+def two_prod(a, b):
+    """a b = p + e with p the fp32 product and e its exact error (both float32)."""
+    a = np.asarray(a, np.float32)
+    b = np.asarray(b, np.float32)
+    p = (a * b).astype(np.float32)
+    e = (a.astype(np.float64) * b.astype(np.float64) - p.astype(np.float64)).astype(np.float32)
+    return p, e
+
+
+def split_df(hi, lo, n):
+    """hi + lo as n bf16 terms, each the nearest bf16 to what remains; lo joins the
+    remainder after the first term (fp32 arithmetic).  Returns the sum of the terms (float64)."""
+    r = np.asarray(hi, np.float32)
+    tot = np.zeros(r.shape)
+    for i in range(n):
+        t = bf16(r)
+        tot = tot + t.astype(np.float64)
+        r = (r - t).astype(np.float32)
+        if i == 0:
+            r = (r + np.asarray(lo, np.float32)).astype(np.float32)
+    return tot
+
+
+def fma32(a, b, c):
+    """fp32 fused multiply-add (one rounding), via float64."""
+    return (np.asarray(a, np.float64) * np.asarray(b, np.float64) + np.asarray(c, np.float64)).astype(np.float32)
+
+
 def kernel_constants(lam: float, sigma: float, d: int = 128):
     """The fp32 constants the launch computes in fp64 and the kernel derives from them."""
     sc = f32(LOG2E / math.sqrt(d))
@@ -58,18 +88,27 @@ def kernel_constants(lam: float, sigma: float, d: int = 128):
 def expansion_terms(ux, uy, xk, yk, lam, sigma, h, w, d: int = 128):
     """The raw-unit bias the K = 16 extension contributes for correspondences (ux, uy)
     [N] against key cells (xk, yk) [M], with every product exact: [N, M] float64.
-    Only the fp32 coefficient roundings and the bf16 splits are modelled; the tensor
-    core's own summation is not."""
+    Modelled: A rounded to two bf16 terms (A'); -2 A' ux', -2 A' uy' and A' (ux'^2 + uy'^2)
+    formed in double-fp32 and split into 4, 4 and 3 bf16 terms; q_k in two terms.  The
+    tensor core's own summation is not."""
     sc, coef, inv_sc = kernel_constants(lam, sigma, d)
     xc, yc = f32(0.5) * f32(w - 1), f32(0.5) * f32(h - 1)
     A = f32(coef * inv_sc)
+    ah = bf16(A)
+    al = bf16(np.float32(A - ah))
     ux_ = (np.asarray(ux, np.float32) - xc).astype(np.float32)
     uy_ = (np.asarray(uy, np.float32) - yc).astype(np.float32)
-    c0 = split3(np.full(ux_.shape, A, np.float32))
-    c1 = split3((f32(-2.0) * A * ux_).astype(np.float32))
-    c2 = split3((f32(-2.0) * A * uy_).astype(np.float32))
-    fm = (ux_.astype(np.float64) * ux_ + (uy_ * uy_).astype(np.float32)).astype(np.float32)  # fmaf(ux, ux, uy*uy)
-    c3 = split3((A * fm).astype(np.float32))
+    p, e = two_prod(np.full(ux_.shape, ah, np.float32), ux_)
+    c1 = split_df((f32(-2.0) * p).astype(np.float32), (f32(-2.0) * fma32(al, ux_, e)).astype(np.float32), 4)
+    p, e = two_prod(np.full(uy_.shape, ah, np.float32), uy_)
+    c2 = split_df((f32(-2.0) * p).astype(np.float32), (f32(-2.0) * fma32(al, uy_, e)).astype(np.float32), 4)
+    sx, ex = two_prod(ux_, ux_)
+    sy, ey = two_prod(uy_, uy_)
+    sq = (sx + sy).astype(np.float32)  # two_sum: the exact error of the fp32 sum
+    es = (sx.astype(np.float64) + sy.astype(np.float64) - sq.astype(np.float64)).astype(np.float32)
+    sl = ((ex + ey).astype(np.float32) + es).astype(np.float32)
+    p, e = two_prod(np.full(sq.shape, ah, np.float32), sq)
+    c3 = split_df(p, fma32(ah, sl, fma32(al, sq, e)), 3)
     xr = (np.asarray(xk, np.float64) - float(xc))
     yr = (np.asarray(yk, np.float64) - float(yc))
     q = xr * xr + yr * yr
@@ -77,7 +116,17 @@ def expansion_terms(ux, uy, xk, yk, lam, sigma, h, w, d: int = 128):
     ql = bf16((q - qh).astype(np.float32)).astype(np.float64)
     xb = bf16(xr.astype(np.float32)).astype(np.float64)
     yb = bf16(yr.astype(np.float32)).astype(np.float64)
-    return (c0[:, None] * (qh + ql)[None] + c1[:, None] * xb[None] + c2[:, None] * yb[None] + c3[:, None])
+    a = float(ah) + float(al)
+    return (a * (qh + ql)[None] + c1[:, None] * xb[None] + c2[:, None] * yb[None] + c3[:, None])
+
+
+def strength(lam, sigma, d: int = 128):
+    """The bias strength the expansion applies, A' (two bf16 terms of A), over the exact
+    lambda sqrt(d) / (2 sigma^2): the consistent scale of the tensor core's bias."""
+    sc, coef, inv_sc = kernel_constants(lam, sigma, d)
+    A = f32(coef * inv_sc)
+    ah = bf16(A)
+    return (float(ah) + float(bf16(np.float32(A - ah)))) / (-lam * math.sqrt(d) / (2.0 * sigma * sigma))
 
 
 def exact_bias_raw(ux, uy, xk, yk, lam, sigma, d: int = 128):
