@@ -246,24 +246,31 @@ E2E_INPUTS = ("q", "k_new", "v_new", "depth")
 
 
 E2E_BUFFERS = 3
+# blocks of the SM-issued copies: eight 1024-thread blocks reach the host link's rate
+E2E_COPY_BLOCKS = 8
 
 
-def run_e2e(W, stream, steps: int):
+def run_e2e(W, stream, steps: int, nb: int = None, copy: str = "sm"):
     """The step through the public API with host buffers, pipelined against one copy stream.
 
     Every step copies its inputs (Q, the new chunk's K/V, its depth) from pinned host
     memory and copies O back, on one copy stream: the step's copies fit in its kernel
     time one direction at a time, and running both directions at once made the host
     side slow and erratic.  NB device buffer sets let the uploads run up to NB - 1 steps
-    ahead and the downloads trail, overlapping the kernels.  Returns (seconds per step,
-    h2d, d2h bytes)."""
+    ahead and the downloads trail, overlapping the kernels.
+    copy = "sm": the copies are crc_host_copy launches (SM-issued over the host link) on
+    a high-priority stream, so that their blocks start beside the attention kernel;
+    copy = "ce": cudaMemcpyAsync on the copy engines.
+    Returns (seconds per step, h2d, d2h bytes, timeline)."""
     import torch
 
-    NB = E2E_BUFFERS
+    from paper_2607_21848_gb300 import api
+
+    NB = nb or E2E_BUFFERS
     host_in = {k: W[k].cpu().pin_memory() for k in E2E_INPUTS}
     dev = [W] + [dict(W, **{k: torch.empty_like(W[k]) for k in E2E_INPUTS + ("o",)}) for _ in range(NB - 1)]
     host_out = [torch.empty(W["o"].shape, dtype=W["o"].dtype, pin_memory=True) for _ in range(NB)]
-    h2d_s = torch.cuda.Stream()
+    h2d_s = torch.cuda.Stream(priority=-1) if copy == "sm" else torch.cuda.Stream()
     d2h_s = h2d_s  # one copy stream for both directions
     in_ready = [torch.cuda.Event() for _ in range(NB)]
     done = [torch.cuda.Event() for _ in range(NB)]
@@ -288,7 +295,10 @@ def run_e2e(W, stream, steps: int):
                 h2d_s.wait_event(done[b])  # step i-NB has finished reading buffer b
             up[i][0].record(h2d_s)
             for k in E2E_INPUTS:
-                dev[b][k].copy_(host_in[k], non_blocking=True)
+                if copy == "sm":
+                    api.crc_host_copy(dev[b][k], host_in[k], stream=h2d_s, blocks=E2E_COPY_BLOCKS)
+                else:
+                    dev[b][k].copy_(host_in[k], non_blocking=True)
             up[i][1].record(h2d_s)
             in_ready[b].record(h2d_s)
 
@@ -308,7 +318,10 @@ def run_e2e(W, stream, steps: int):
         with torch.cuda.stream(d2h_s):
             d2h_s.wait_event(done[b])
             dn[i][0].record(d2h_s)
-            host_out[b].copy_(dev[b]["o"], non_blocking=True)
+            if copy == "sm":
+                api.crc_host_copy(host_out[b], dev[b]["o"], stream=d2h_s, blocks=E2E_COPY_BLOCKS)
+            else:
+                host_out[b].copy_(dev[b]["o"], non_blocking=True)
             dn[i][1].record(d2h_s)
             out_read[b].record(d2h_s)
     stream.wait_stream(h2d_s)
@@ -908,8 +921,12 @@ def main():
     barrier()
     with ClockSampler(local) as clk_e2e:
         e2e_s, h2d, d2h, e2e_timeline = run_e2e(W, stream, max(3, args.steps))  # as many steps as the device timing
-    link = link_gbs(W)
     e2e_s = max_over_ranks(e2e_s, world, device)
+    barrier()
+    # the same pipeline with the copies on the copy engines, for comparison
+    ce_s, _, _, ce_timeline = run_e2e(W, stream, max(3, args.steps), copy="ce")
+    ce_s = max_over_ranks(ce_s, world, device)
+    link = link_gbs(W)
     graph_s = run_graph(W, max(3, min(args.steps, 20)))
     context = sdpa_context(W, alg["flops"]) if not args.no_context else None
     sweep = shapes = modes = stream_ctx = gsweep = None
@@ -984,10 +1001,19 @@ def main():
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
                 "pipelining": f"{E2E_BUFFERS} device buffer sets; on one copy stream, uploads run up to "
                               f"{E2E_BUFFERS - 1} steps ahead and downloads trail, overlapping the kernels",
+                "copies": f"crc_host_copy ({E2E_COPY_BLOCKS} blocks of 1024 threads, SM-issued over the host "
+                          "link) on a high-priority stream",
+                "gpu_launches_per_step": LAUNCHES_PER_STEP + len(E2E_INPUTS) + 1,
                 "link_gbs": link,
                 "timeline": e2e_timeline,
                 "clocks": clk_e2e.summary(),
-                "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6},
+                "copy_ms_per_step": (h2d / link["h2d"] + d2h / link["d2h"]) / 1e6,
+                "copy_engines": {"value": whole_job_tflops(alg["flops"], ce_s, world), "ms_per_step": ce_s * 1e3,
+                                 "note": "the same pipeline with cudaMemcpyAsync on the copy engines",
+                                 "upload_ms": ce_timeline["upload_ms"], "upload_ms_max": ce_timeline["upload_ms_max"],
+                                 "download_ms_max": ce_timeline["download_ms_max"],
+                                 "compute_ms": ce_timeline["compute_ms"],
+                                 "compute_gap_total_ms": ce_timeline["compute_gap_total_ms"]}},
         "graph": {"ms_per_step": graph_s * 1e3, "eager_ms_per_step": step_s * 1e3,
                   "note": "one step captured in a CUDA graph and replayed"},
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,

@@ -481,6 +481,33 @@ typedef struct {
  */
 crc_status crc_chunk_step(const crc_step_plan* plan, const crc_step* d_step, cudaStream_t s);
 
+/*
+ * crc_host_copy — copies `bytes` bytes from src to dst with the GPU's SMs: how a
+ * step's host-resident inputs (Q, the new chunk's K/V, its depth) reach the GPU and
+ * its output O returns.  (The paper has no counterpart; Sec. 4.2-4.3 define the step
+ * these copies feed.)
+ *
+ * On GB300 the GPU reaches page-locked host memory directly over the coherent CPU-GPU
+ * link, so a kernel moves host data at the link's own rate (about 210 GB/s to the
+ * device and 190 GB/s back, measured) without the copy engines; eight SMs suffice for
+ * that rate.  On some machines the copy engines stall for 35-100 ms at a time;
+ * copies issued by the SMs were not seen to stall.  The copy runs `blocks` blocks of
+ * 1024 threads (0 = 8), each resident on one SM until it ends.  To run it beside a
+ * kernel that fills the GPU, enqueue it on a stream of higher priority: at equal
+ * priority its blocks wait until the earlier kernel has dispatched all of its own.
+ *
+ * src, dst: device memory of the current device, page-locked host memory (allocated
+ *   or registered with CUDA) or managed memory, in any combination; both 16-byte
+ *   aligned; the two ranges must not overlap.  bytes: any size.
+ * Returns CRC_OK (0 bytes: nothing enqueued); CRC_ERR_INVALID_ARG for a null pointer,
+ * blocks outside 0..4096, overlapping ranges, or a range the device cannot reach in
+ * one contiguous mapping (pageable host memory, another device's memory, a range that
+ * runs past its allocation into unmapped memory), all found before anything is
+ * enqueued; CRC_ERR_UNSUPPORTED for a pointer that is not 16-byte aligned;
+ * CRC_ERR_CUDA when the launch fails.
+ */
+crc_status crc_host_copy(void* dst, const void* src, size_t bytes, int32_t blocks, cudaStream_t s);
+
 /* Bound on the error of the tensor-core expansion of the Eq. 2 bias on an h x w grid,
  * in base-2 logit units: 2^-24 lambda log2(e) / (2 sigma^2) (w^2 + h^2), besides the
  * consistent 2^-17 scale of the bias strength; +inf where

@@ -123,6 +123,7 @@ _SIGS = {
                                          C.c_int32, C.c_void_p, C.c_void_p]),
     "crc_bias_expansion_bound": (C.c_double, [C.c_float, C.c_float, C.c_int32, C.c_int32]),
     "crc_chunk_step": (C.c_int32, [_P(crc_step_plan), C.c_void_p, C.c_void_p]),
+    "crc_host_copy": (C.c_int32, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_int32, C.c_void_p]),
 }
 
 EXPORTED = tuple(_SIGS)

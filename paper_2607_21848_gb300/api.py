@@ -247,6 +247,18 @@ def crc_gather(shp: _abi.crc_shape, pool: torch.Tensor, idx: torch.Tensor, k: in
                               C.byref(rope) if rope is not None else None, _stream(stream)))
 
 
+def crc_host_copy(dst: torch.Tensor, src: torch.Tensor, stream=None, blocks: int = 0) -> None:
+    """Copy src into dst (same number of bytes, both contiguous) with the GPU's SMs;
+    either side may be a CUDA tensor or a pinned CPU tensor."""
+    lib = _abi.load()
+    if not (dst.is_contiguous() and src.is_contiguous()):
+        raise ValueError("expected contiguous tensors")
+    nbytes = dst.numel() * dst.element_size()
+    if nbytes != src.numel() * src.element_size():
+        raise ValueError("dst and src differ in size")
+    _abi.check("crc_host_copy", lib.crc_host_copy(dst.data_ptr(), src.data_ptr(), nbytes, blocks, _stream(stream)))
+
+
 def crc_correspond(shp: _abi.crc_shape, cur_frames: np.ndarray, depth: torch.Tensor, bank: Bank, idx: torch.Tensor,
                    count: Optional[torch.Tensor], k: int, eps: float, uv: torch.Tensor, cell: Optional[torch.Tensor],
                    valid: torch.Tensor, stream=None) -> None:

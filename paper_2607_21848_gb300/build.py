@@ -15,7 +15,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libcrc.so")
-SOURCES = ["api.cu", "bank.cu", "retrieve.cu", "correspond.cu", "attn_simt.cu", "attn_tc.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "bank.cu", "retrieve.cu", "correspond.cu", "attn_simt.cu", "attn_tc.cu", "noalloc.cu", "host_copy.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-cudart", "shared", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 

@@ -536,3 +536,7 @@ double crc_bias_expansion_bound(float lambda, float sigma, int32_t h, int32_t w)
 }
 
 }  // extern "C"
+
+namespace crc {
+crc_status record_cuda_error(cudaError_t e) { return cuda_fail(e); }
+}  // namespace crc

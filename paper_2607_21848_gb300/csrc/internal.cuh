@@ -8,6 +8,10 @@
 
 namespace crc {
 
+// Records e as the calling thread's last CUDA error (crc_last_cuda_error) and
+// returns CRC_ERR_CUDA: for entry points defined outside api.cu.
+crc_status record_cuda_error(cudaError_t e);
+
 // One crc_frame record is 21 doubles: K[9], R[9], c[3].
 constexpr int kFrameDoubles = 21;
 

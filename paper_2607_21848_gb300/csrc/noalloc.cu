@@ -52,7 +52,7 @@ extern "C" crc_status crc_retrieve_noalloc(const crc_bank* bank, int32_t bank_co
   void* scratch = nullptr;
   if (need > 0) {
     const cudaError_t e = scratch_address(&scratch);
-    if (e != cudaSuccess) return CRC_ERR_CUDA;
+    if (e != cudaSuccess) return crc::record_cuda_error(e);
   }
   return crc_retrieve(bank, bank_count, shape, cur, n, p, cache, rope, d_idx, d_score, d_count, scratch,
                       need > 0 ? (size_t)CRC_NOALLOC_SCRATCH_BYTES : 0, s);

@@ -292,3 +292,16 @@ def test_attention_limits_of_the_tensor_core_kernel(lib):
     n_keys = 641 * 128
     segs = [(0, n_keys, _abi.CRC_SEG_WINDOW, 0)]
     assert _attend(lib, cache=_cache(segs, n_keys), k=0, uv=None, valid=None) == UNSUPPORTED
+
+
+@pytest.mark.parametrize("dst, src, nbytes, blocks, status", [
+    (_ptr(1), _ptr(2), 0, 0, OK),                  # nothing to copy: nothing enqueued
+    (None, _ptr(2), 64, 0, INVALID),
+    (_ptr(1), None, 64, 0, INVALID),
+    (_ptr(1), _ptr(2), 64, -1, INVALID),
+    (_ptr(1), _ptr(2), 64, 4097, INVALID),
+    (_ptr(1) + 8, _ptr(2), 64, 0, UNSUPPORTED),    # 16-byte alignment of both pointers
+    (_ptr(1), _ptr(2) + 4, 64, 0, UNSUPPORTED),
+])
+def test_host_copy_rejections_before_any_cuda_call(lib, dst, src, nbytes, blocks, status):
+    assert lib.crc_host_copy(dst, src, nbytes, blocks, None) == status
