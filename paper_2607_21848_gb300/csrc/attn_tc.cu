@@ -312,8 +312,9 @@ constexpr int kBiasGauss = 1;
 constexpr int kBiasDirect = 2;
 
 // MODE: one of the kBias* forms; the tensor-core instantiation carries none of the
-// per-score code.
-template <int MODE>
+// per-score code.  FC: the frame-causal test mode (CRC_ATTN_FRAME_CAUSAL), compiled
+// only into its own instantiations (its per-tile test cost the default kernel 1 %).
+template <int MODE, bool FC>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ TcParams P) {
@@ -394,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (len <= 0) continue;
       const bool ret = sg.kind == CRC_SEG_RETRIEVED;
       // the current chunk's segment is cut per frame too when the frame-causal mask is on
-      const bool curc = sg.kind == CRC_SEG_CURRENT && a.frame_causal;
+      const bool curc = FC && sg.kind == CRC_SEG_CURRENT;
       if (ret && a.slot_chunk && a.slot_chunk[sg.slot] < 0) continue;  // empty slot: masked
       const int nr = (ret || curc) ? a.F : 1;
       for (int rr = 0; rr < nr; ++rr) {
@@ -758,7 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // frame-causal mode: a tile of the current chunk's frame f is invisible to this row when
       // the row's query frame is earlier; its weights are then 2^-inf = 0 and m, l stay put
       bool rowmask = false;
-      if (a.frame_causal) {
+      if constexpr (FC) {
         const int kf1 = tiles[j].kf1;
         rowmask = kf1 > 0 && kf1 - 1 > qframe;
       }
@@ -943,10 +944,16 @@ cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
   P.gauss_gc = (float)((double)a.lambda * sqrt((double)a.d));
   P.gauss_k = (float)(1.4426950408889634 / (2.0 * (double)a.sigma * (double)a.sigma));
   P.timeout_ns = 2000000000ull;
-  auto kernel = a.bias_form == 1 ? attn_tc_kernel<kBiasGauss>
-                : (a.bias_direct || bias_expansion_bound(a.lambda, a.sigma, a.h, a.w) > kExpansionLimit)
-                    ? attn_tc_kernel<kBiasDirect>
-                    : attn_tc_kernel<kBiasTensor>;
+  const int mode = a.bias_form == 1 ? kBiasGauss
+                   : (a.bias_direct || bias_expansion_bound(a.lambda, a.sigma, a.h, a.w) > kExpansionLimit)
+                       ? kBiasDirect
+                       : kBiasTensor;
+  using KernelFn = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const TcParams);
+  static const KernelFn kernels[3][2] = {
+      {attn_tc_kernel<kBiasTensor, false>, attn_tc_kernel<kBiasTensor, true>},
+      {attn_tc_kernel<kBiasGauss, false>, attn_tc_kernel<kBiasGauss, true>},
+      {attn_tc_kernel<kBiasDirect, false>, attn_tc_kernel<kBiasDirect, true>}};
+  const KernelFn kernel = kernels[mode][a.frame_causal ? 1 : 0];
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
   dim3 grid((a.Nq + NQT * BM - 1) / (NQT * BM), a.H, a.L);
