@@ -215,7 +215,7 @@ LAUNCHES_PER_STEP = 5
 # DRAM bytes (read + write) per layer of attn_tc_kernel at the Wan-1.3B chunk shape, from one
 # ncu capture of a 2-layer launch of the current kernel (259.6 + 23.9 MB / 2); traffic grows in
 # proportion to layers.  Valid only for that shape and the kernel version it was captured on.
-ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.72e6}
+ATTN_DRAM_BYTES_PER_LAYER = {(12, 4680, 18720): 141.71e6}
 
 
 # ---------------------------------------------------------------------------- ranks
