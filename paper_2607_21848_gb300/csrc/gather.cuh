@@ -94,6 +94,34 @@ struct Vec16<false> {
   }
 };
 
+// One 16-byte vector of interleaved pairs: the pairs whose bit is set in `rot` are
+// rotated by f[] (as rotate_pair, rounded back to the cache dtype); the others keep
+// their bits exactly.  Every lane runs the same instructions, whatever its pairs.
+template <bool BF16>
+__device__ __forceinline__ uint4 rotate_interleaved(const uint4& v, const float2* f, uint32_t rot) {
+  uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if constexpr (BF16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {  // word i holds pair i
+      float a = __uint_as_float(w[i] << 16), b = __uint_as_float(w[i] & 0xffff0000u);
+      rotate_pair(a, b, f[i]);
+      const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+      const uint32_t nw = *reinterpret_cast<const uint32_t*>(&h);
+      w[i] = ((rot >> i) & 1u) ? nw : w[i];
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {  // words 2i, 2i + 1 hold pair i
+      float a = __uint_as_float(w[2 * i]), b = __uint_as_float(w[2 * i + 1]);
+      rotate_pair(a, b, f[i]);
+      const bool on = ((rot >> i) & 1u) != 0;
+      w[2 * i] = on ? __float_as_uint(a) : w[2 * i];
+      w[2 * i + 1] = on ? __float_as_uint(b) : w[2 * i + 1];
+    }
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // One key row (H heads of d channels) copied by a warp with the temporal pairs of
 // every head rotated by cs[i].  Interleaved pairs lie inside one 16-byte vector
 // (channel0 is even).  Half-split pairs (c, c + pairs) lie in two vectors `half`
@@ -118,6 +146,32 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
   const int vph = g.d / N;  // vectors per head
   const int c0 = g.rope_c0, np = g.rope_pairs, np2 = 2 * g.rope_pairs;
   const int half = np / N;
+  if ((32 % vph) == 0 && g.rope_interleaved) {
+    // interleaved pairs, lane l meeting the same channels in every head: the row is
+    // copied like a plain row, four vectors in flight per lane, each passed through
+    // the lane's fixed rotation (a no-op select on lanes without rotated pairs)
+    const int ch = (lane % vph) * N;
+    constexpr int NP = N / 2;
+    uint32_t rot = 0u;
+    float2 f[NP];
+#pragma unroll
+    for (int i = 0; i < NP; ++i) {
+      const int che = ch + 2 * i;
+      const bool in = che >= c0 && che < c0 + np2;
+      rot |= in ? (1u << i) : 0u;
+      f[i] = in ? cs[(che - c0) >> 1] : make_float2(1.f, 0.f);
+    }
+    int c = lane;
+    for (; c + 96 < n; c += 128) {
+      const uint4 a0 = __ldg(s + c), a1 = __ldg(s + c + 32), a2 = __ldg(s + c + 64), a3 = __ldg(s + c + 96);
+      d[c] = rotate_interleaved<BF16>(a0, f, rot);
+      d[c + 32] = rotate_interleaved<BF16>(a1, f, rot);
+      d[c + 64] = rotate_interleaved<BF16>(a2, f, rot);
+      d[c + 96] = rotate_interleaved<BF16>(a3, f, rot);
+    }
+    for (; c < n; c += 32) d[c] = rotate_interleaved<BF16>(__ldg(s + c), f, rot);
+    return;
+  }
   if ((32 % vph) == 0) {
     const int ch = (lane % vph) * N;
     const int kind = g.rope_interleaved ? ((ch + N > c0 && ch < c0 + np2) ? 1 : 0)

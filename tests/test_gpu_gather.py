@@ -114,6 +114,32 @@ def test_rope_repositioning_matches_oracle(dtype):
         assert bool((cache.k[:, 3 * Nc:4 * Nc] == -3.0).all())
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_unrotated_pairs_keep_their_bits_next_to_rotated_ones(dtype):
+    """A temporal block that starts and ends inside 16-byte vectors (channels 2-19): the
+    pairs it does not cover in those vectors (channels 0-1 and 20-23) must keep their bits,
+    even for -0, infinities, NaN and subnormals, which a rotation by angle 0 would not."""
+    d = 64
+    cache, pool, shp, Nc = _setup(dtype, d=d)
+    specials = torch.tensor([-0.0, float("inf"), float("-inf"), float("nan"), -1e-40, 0.0, -3.5, 1e30])
+    k = pool[:, 0]
+    for n, ch in enumerate([0, 1, 20, 21, 22, 23]):
+        k[..., ch] = specials.roll(n)[torch.arange(k[..., ch].numel()) % len(specials)].reshape(k[..., ch].shape).to(dtype).cuda()
+    rope = api.rope_params(2, 9, 500.0, True, pos_slot0=-5, pos_stride=3, frame_pos0=7)
+    chunks = [11, 3, -1]
+    api.crc_gather(shp, pool, torch.tensor(chunks, dtype=torch.int32, device="cuda"), 3, cache, rope=rope)
+    torch.cuda.synchronize()
+    ibits = torch.int16 if dtype == torch.bfloat16 else torch.int32
+    for r in (0, 1):
+        seg = slice((1 + r) * Nc, (2 + r) * Nc)
+        got = cache.k[:, seg].contiguous().view(ibits)
+        src = pool[chunks[r] % pool.shape[0], 0].contiguous().view(ibits)
+        outside = [0, 1] + list(range(20, d))
+        assert torch.equal(got[..., outside], src[..., outside])
+        # and the block itself was moved: its bits differ from the slab's
+        assert not torch.equal(got[..., 2:20], src[..., 2:20])
+
+
 def test_zero_shift_is_a_plain_copy():
     # slot 0 holding chunk 5 at pos_slot0 = frame_pos0 + 5 F is not moved: byte-exact
     dtype = torch.bfloat16
