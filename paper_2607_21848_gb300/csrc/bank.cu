@@ -87,9 +87,11 @@ __global__ void __launch_bounds__(256) cache_update_kernel(const __grid_constant
     const int t = (int)(rem - (int64_t)l * a.Nc);
     const char* src = (kv ? a.v_src : a.k_src) + rem * a.row_bytes;
     char* dst = slab + kv * half + rem * a.row_bytes;
-    char* win = nullptr;
-    if (win_k) win = (kv ? win_v : win_k) + l * a.win_layer_stride + t * a.win_token_stride;
-    warp_copy_row(src, dst, win, a.row_bytes, lane);
+    if (win_k)
+      warp_copy_row<2>(src, dst, (kv ? win_v : win_k) + l * a.win_layer_stride + t * a.win_token_stride, a.row_bytes,
+                       lane);
+    else
+      warp_copy_row<1>(src, dst, nullptr, a.row_bytes, lane);
   }
 }
 

