@@ -3,6 +3,7 @@
   python sweeps.py correspond      # 126 MB reprojection sweep, scene depth
   python sweeps.py correspond-iid  # the same with depth drawn per token
   python sweeps.py gather          # crc_gather, plain and re-positioned
+  python sweeps.py retrieve        # Eq. 1 scoring and top-k over banks of 64 to 261 120 entries
 
 Measurement tooling beside bench.py (which imports it for its context block); not part
 of the library package.
@@ -132,6 +133,57 @@ def gather_sweep(device="cuda:0", iters: int = 10):
     return out
 
 
+def retrieve_sweep(device="cuda:0", iters: int = 20):
+    """Eq. 1 scoring and top-k alone (no gather) over banks from 64 to 261 120 entries,
+    at k = 1 and k = 8: the bank's chunk poses are drawn at random, every entry is
+    admissible (E = 1, no centre or view gate, delta = 1), so every entry is scored and
+    merged.  Through the workspace call and through crc_retrieve_noalloc."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2607_21848_gb300 import _abi, api
+
+    F, h, w = 3, 30, 52
+    walk = synth.random_walk(synth.rng(7, "sweep"), 1, F, synth.pinhole(h, w, 90.0), step=0.5, radius=24.0)
+    cur = synth.frame_records(walk[0])
+    out = {}
+    for B in (64, 2000, 20000, 100003, 261120):
+        bank = api.Bank(B, F, h, w, 1, 1, 64, torch.float32, 1, device=device, with_kv=False)
+        g = np.random.default_rng(B)
+        c = g.normal(size=(B, 3)) * 20.0
+        v = g.normal(size=(B, 3))
+        v /= np.linalg.norm(v, axis=1, keepdims=True)
+        bank.centre.copy_(torch.from_numpy(c))
+        bank.view.copy_(torch.from_numpy(v))
+        shp = api.shape(1, 1, 64, F, h, w, torch.float32)
+        row = {}
+        for k in (1, 8):
+            params = api.retrieval_params(1.0, 0.5, float("inf"), -1.0, 1, k)
+            idx = torch.empty(k, dtype=torch.int32, device=device)
+            cnt = torch.empty(1, dtype=torch.int32, device=device)
+            calls = {"workspace": lambda: api.crc_retrieve(bank, B, shp, cur, B, params, None, idx, None, cnt)}
+            if _abi.load().crc_retrieve_workspace_size(B, k) <= _abi.CRC_NOALLOC_SCRATCH_BYTES:
+                calls["noalloc"] = lambda: api.crc_retrieve_noalloc(bank, B, shp, cur, B, params, None, idx, None, cnt)
+            got = {}
+            for name, fn in calls.items():
+                fn()
+                torch.cuda.synchronize()
+                got[name] = idx.cpu().clone()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                for _ in range(iters):
+                    fn()
+                e1.record()
+                torch.cuda.synchronize()
+                row[f"k{k}_{name}_us"] = e0.elapsed_time(e1) / iters * 1e3
+            assert all(torch.equal(x, got["workspace"]) for x in got.values()), "noalloc and workspace calls disagree"
+            assert int(cnt.item()) == min(k, B)
+        out[str(B)] = row
+    return out
+
+
 def main(argv=None):
     argv = sys.argv[1:] if argv is None else argv
     what = argv[0] if argv else "correspond"
@@ -147,6 +199,8 @@ def main(argv=None):
         print(json.dumps(correspond_sweep("cuda:0", depth="iid")))
     elif what == "gather":
         print(json.dumps(gather_sweep("cuda:0")))
+    elif what == "retrieve":
+        print(json.dumps(retrieve_sweep("cuda:0")))
     else:
         raise SystemExit(f"unknown sweep {what}")
 
